@@ -1,0 +1,170 @@
+/*
+ * libarcher -- the per-step hot path of Archer's asymmetric-cache denoising
+ * step (Adaptive Reuse of Cached Hidden States for Efficient Rollback,
+ * arXiv 2608.08086) for one NVIDIA GB300 (sm_103a).
+ *
+ * Plain C ABI: device pointers, sizes and a CUDA stream.  No call allocates
+ * device memory, synchronises the device or prints.  Every call is
+ * asynchronous on `stream` (a cudaStream_t passed as void*; NULL = the legacy
+ * default stream) and returns an archer_status.  A non-zero status means that
+ * nothing was launched, except ARCHER_ERR_CUDA from a failed launch; the
+ * reason is available from archer_last_error() on the calling thread.
+ *
+ * Layouts (all contiguous, row-major, bf16 = IEEE bfloat16 bit patterns):
+ *   queries  [B, M, Hq,  D]     M = G (cached step) or N = P + G (refresh)
+ *   prompt   [B, P, Hkv, D]     K and V separately (the cache C_p, Sec. 4.1)
+ *   response [B, G, Hkv, D]     K and V separately
+ *   output   [B, M, Hq,  D]     bf16;  lse [B, Hq, M] fp32 (natural log)
+ * Every device pointer must be 16-byte aligned; D must be 64 or 128;
+ * Hq % Hkv == 0 (GQA: query head h reads KV head h / (Hq / Hkv)).
+ */
+#ifndef ARCHER_H_
+#define ARCHER_H_
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum archer_status {
+  ARCHER_OK = 0,
+  ARCHER_ERR_ARG = -1,          /* null pointer, negative size, misalignment  */
+  ARCHER_ERR_UNSUPPORTED = -2,  /* valid but unsupported shape (e.g. D = 96)   */
+  ARCHER_ERR_CUDA = -3,         /* a CUDA runtime/driver call failed          */
+  ARCHER_ERR_TIMEOUT = -4       /* a kernel's bounded wait expired            */
+} archer_status;
+
+typedef enum archer_dtype {
+  ARCHER_DTYPE_BF16 = 0,
+  ARCHER_DTYPE_F32 = 1
+} archer_dtype;
+
+/* Problem statement of one attention layer (Sec. 4.1: prompt p of length P,
+ * response g of length G, N = P + G).  softmax_scale <= 0 selects
+ * 1/sqrt(head_dim). */
+typedef struct archer_shape {
+  int batch;        /* B  >= 0                                */
+  int prompt_len;   /* P  >= 0 (P = 0: response-only attention) */
+  int resp_len;     /* G  >= 1                                */
+  int n_heads;      /* Hq >= 1                                */
+  int n_kv_heads;   /* Hkv >= 1, Hq % Hkv == 0                */
+  int head_dim;     /* D in {64, 128}                         */
+  float softmax_scale;
+} archer_shape;
+
+/*
+ * Cached response step -- Sec. 4.1, Eq. archer-cached and Eq. archer-attention:
+ *   out = Attn(Q_g(g_t), [K_p(g_r) || K_g(g_t)], [V_p(g_r) || V_g(g_t)])
+ * Non-causal: each of the G response queries attends to all P cached prompt
+ * keys and all G fresh response keys; the concatenation is never formed.
+ *   q_resp  [B, G, Hq, D]  bf16     k_cache, v_cache [B, P, Hkv, D] bf16 (read)
+ *   k_resp, v_resp [B, G, Hkv, D] bf16
+ *   out     [B, G, Hq, D]  bf16 (written)
+ *   lse     [B, Hq, G] fp32 (written; may be NULL)
+ *   workspace / ws_bytes: scratch of at least archer_attn_workspace_size()
+ *   bytes (may be NULL when that size is 0).  Owned by the caller; must not be
+ *   used by another call that can overlap on the GPU.
+ * k_cache/v_cache may be NULL only when P == 0.
+ */
+int archer_attn_step(const archer_shape* shape, const void* q_resp, const void* k_cache,
+                     const void* v_cache, const void* k_resp, const void* v_resp, void* out,
+                     float* lse, void* workspace, size_t ws_bytes, void* stream);
+
+/*
+ * Prompt refresh -- Sec. 4.2 and Algorithm 1's FullForward: every position of
+ * a refreshed sequence is a query over the fresh [K_p(g_t) || K_g(g_t)], and
+ * the prompt cache is replaced by the fresh prompt K/V (C_r <- C_p(g_t)).
+ *   q_all [B, N, Hq, D] bf16 (rows 0..P-1 prompt queries, P..N-1 response queries)
+ *   k_prompt_new, v_prompt_new [B, P, Hkv, D] bf16: fresh prompt K/V
+ *   k_resp, v_resp [B, G, Hkv, D] bf16
+ *   out [B, N, Hq, D] bf16; lse [B, Hq, N] fp32 (may be NULL)
+ *   k_cache, v_cache [B, P, Hkv, D] bf16: for a refreshed sequence overwritten
+ *     with k_prompt_new / v_prompt_new (no copy when the pointers are equal);
+ *     for a sequence whose flag is clear, read as the anchored cache.
+ *   refresh_flags [B] uint8 (device; may be NULL = refresh every sequence).
+ *     A sequence whose flag is 0 takes the cached step instead: its rows
+ *     P..N-1 of out/lse get Attn(Q_g, [K_cache || K_g], ...), its rows 0..P-1
+ *     are left untouched and its cache is kept.  This serves a batch with
+ *     per-sequence refresh decisions in one call.
+ */
+int archer_prompt_refresh(const archer_shape* shape, const void* q_all, const void* k_prompt_new,
+                          const void* v_prompt_new, const void* k_resp, const void* v_resp,
+                          void* out, float* lse, void* k_cache, void* v_cache,
+                          const uint8_t* refresh_flags, void* workspace, size_t ws_bytes,
+                          void* stream);
+
+/* Scratch bytes archer_attn_step / archer_prompt_refresh need for n_queries
+ * (= G or N) query rows per sequence; 0 when none is needed. */
+size_t archer_attn_workspace_size(const archer_shape* shape, int n_queries);
+
+/*
+ * Decoder scoring -- the inputs of the rollback decoder's confidence rule
+ * (Sec. 6 "confidence"; the decision margin of Eq. theory-margin is taken on
+ * these probabilities).  For each of the batch * resp_len rows of logits z:
+ *   p        = softmax(z) in fp32
+ *   top1     = the lowest index attaining max_j z_j
+ *   max_prob = p[top1]
+ *   margin   = p[top1] - p[top2], top2 the next index in (value desc, index
+ *              asc) order (margin 0 on a tie; = max_prob when vocab == 1)
+ *   cur_prob = p[cur_tokens[r]] where mask_state[r] == 0 and
+ *              0 <= cur_tokens[r] < vocab, else 0   (skipped when NULL)
+ *   logits:   [batch * resp_len rows, row_stride elements], dtype bf16 or f32,
+ *             row_stride >= vocab; the row stride in bytes must be a multiple
+ *             of 16.  -inf entries have probability 0; NaN gives undefined
+ *             results.  A row with no finite entry is undefined.
+ *   mask_state [rows] uint8 (may be NULL = unmasked); cur_tokens [rows] int32
+ *   (may be NULL); outputs [rows] fp32 / int32 device arrays.
+ *   workspace: at least archer_decode_scores_workspace_size(rows, vocab) bytes,
+ *   zero-filled before its first use; every call leaves it zero-filled again.
+ */
+int archer_decode_scores(int batch, int resp_len, int vocab, int dtype, const void* logits,
+                         int64_t row_stride, const uint8_t* mask_state, const int32_t* cur_tokens,
+                         float* max_prob, int32_t* top1, float* margin, float* cur_prob,
+                         void* workspace, size_t ws_bytes, void* stream);
+
+size_t archer_decode_scores_workspace_size(int rows, int vocab);
+
+/*
+ * Refresh rule -- Sec. 4.2, Eq. archer-distance and Eq. archer-controller,
+ * with the cache-age signal A_t = t - r of Sec. 6 as an optional cap:
+ *   age_t   = age[b] + 1           (denoising steps since the anchor, this one included)
+ *   dist[b] = D_t = sum_i [g_cur[b, i] != g_anchor[b, i]]
+ *   flag[b] = D_t >= K  or  (max_age > 0 and age_t >= max_age)
+ * With update_anchor != 0 a flagged sequence gets g_anchor <- g_cur and
+ * age <- 0 (g_r <- g_t in Algorithm 1), an unflagged one age <- age_t.
+ * With update_anchor == 0 only dist_out and flag_out are written.
+ *   g_cur, g_anchor [batch, resp_len] int32 (token ids; a mask id is just
+ *   another value); age [batch] int32; dist_out [batch] int32 (may be NULL);
+ *   flag_out [batch] uint8.  K = INT32_MAX never refreshes on distance.
+ */
+int archer_should_refresh(int batch, int resp_len, const int32_t* g_cur, int32_t* g_anchor,
+                          int32_t* age, int K, int max_age, int update_anchor, int32_t* dist_out,
+                          uint8_t* flag_out, void* stream);
+
+/* Bit-exact copy of a refreshed sequence's prompt K/V into the cache
+ * (the cache rewrite C_r <- C_p(g_t) of Algorithm 1) for sequences whose flag
+ * is set (all when flags is NULL).  src/dst [B, P, Hkv, D] bf16. */
+int archer_cache_rewrite(const archer_shape* shape, const void* k_src, const void* v_src,
+                         void* k_dst, void* v_dst, const uint8_t* refresh_flags, void* stream);
+
+/* Reads and clears the device-side error word that kernels set when a
+ * bounded wait expires.  Synchronises `stream`.  Returns ARCHER_OK or
+ * ARCHER_ERR_TIMEOUT (or ARCHER_ERR_CUDA). */
+int archer_check_device(void* stream);
+
+/* Human-readable text for a status code (static storage). */
+const char* archer_status_string(int status);
+
+/* Detail of the last failed call on this thread ("" if none). */
+const char* archer_last_error(void);
+
+/* Library version: major * 10000 + minor * 100 + patch. */
+int archer_version(void);
+
+#ifdef __cplusplus
+}  /* extern "C" */
+#endif
+
+#endif  /* ARCHER_H_ */

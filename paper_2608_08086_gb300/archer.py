@@ -1,0 +1,255 @@
+"""Python binding of libarcher's C ABI (include/archer.h), via ctypes.
+
+Argument marshalling only: each function checks dtypes, shapes and devices of
+the torch tensors it is given, passes their device pointers, sizes and the
+current CUDA stream to the C function of the same name, and raises
+ArcherError on a non-zero status.  Every step of the computation runs in
+libarcher's CUDA kernels; there is no fallback path, and importing this
+module fails loudly when libarcher.so is missing.
+"""
+from __future__ import annotations
+
+import ctypes
+import math
+import os
+
+import torch
+
+_PKG = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_PKG, "libarcher.so")
+
+ARCHER_OK = 0
+ARCHER_ERR_ARG = -1
+ARCHER_ERR_UNSUPPORTED = -2
+ARCHER_ERR_CUDA = -3
+ARCHER_ERR_TIMEOUT = -4
+ARCHER_DTYPE_BF16 = 0
+ARCHER_DTYPE_F32 = 1
+K_INFINITE = 2**31 - 1
+
+
+class ArcherError(RuntimeError):
+    def __init__(self, status: int, detail: str):
+        super().__init__(f"archer status {status}: {detail}")
+        self.status = status
+
+
+class archer_shape(ctypes.Structure):
+    _fields_ = [("batch", ctypes.c_int), ("prompt_len", ctypes.c_int), ("resp_len", ctypes.c_int),
+                ("n_heads", ctypes.c_int), ("n_kv_heads", ctypes.c_int), ("head_dim", ctypes.c_int),
+                ("softmax_scale", ctypes.c_float)]
+
+
+def _load():
+    if not os.path.exists(LIB_PATH):
+        raise ImportError(f"{LIB_PATH} is missing: build it with paper_2608_08086_gb300.build.build() "
+                          "(there is no CPU fallback)")
+    L = ctypes.CDLL(LIB_PATH)
+    vp, i, sz = ctypes.c_void_p, ctypes.c_int, ctypes.c_size_t
+    sp = ctypes.POINTER(archer_shape)
+    L.archer_attn_step.argtypes = [sp, vp, vp, vp, vp, vp, vp, vp, vp, sz, vp]
+    L.archer_prompt_refresh.argtypes = [sp, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, sz, vp]
+    L.archer_attn_workspace_size.argtypes = [sp, i]
+    L.archer_attn_workspace_size.restype = sz
+    L.archer_decode_scores.argtypes = [i, i, i, i, vp, ctypes.c_int64, vp, vp, vp, vp, vp, vp, vp, sz, vp]
+    L.archer_decode_scores_workspace_size.argtypes = [i, i]
+    L.archer_decode_scores_workspace_size.restype = sz
+    L.archer_should_refresh.argtypes = [i, i, vp, vp, vp, i, i, i, vp, vp, vp]
+    L.archer_cache_rewrite.argtypes = [sp, vp, vp, vp, vp, vp, vp]
+    L.archer_check_device.argtypes = [vp]
+    L.archer_status_string.argtypes = [i]
+    L.archer_status_string.restype = ctypes.c_char_p
+    L.archer_last_error.argtypes = []
+    L.archer_last_error.restype = ctypes.c_char_p
+    L.archer_version.argtypes = []
+    for name in ("archer_attn_step", "archer_prompt_refresh", "archer_decode_scores", "archer_should_refresh",
+                 "archer_cache_rewrite", "archer_check_device", "archer_version"):
+        getattr(L, name).restype = ctypes.c_int
+    return L
+
+
+lib = _load()
+
+
+def _raise(status: int):
+    if status != ARCHER_OK:
+        raise ArcherError(status, f"{lib.archer_status_string(status).decode()}: {lib.archer_last_error().decode()}")
+
+
+def _stream(stream):
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return ctypes.c_void_p(stream.cuda_stream if hasattr(stream, "cuda_stream") else int(stream))
+
+
+def _ptr(t, dtype=None, what=""):
+    if t is None:
+        return None
+    if not isinstance(t, torch.Tensor) or not t.is_cuda:
+        raise TypeError(f"{what} must be a CUDA tensor")
+    if dtype is not None and t.dtype != dtype:
+        raise TypeError(f"{what} must be {dtype}, got {t.dtype}")
+    if not t.is_contiguous():
+        raise ValueError(f"{what} must be contiguous")
+    return ctypes.c_void_p(t.data_ptr())
+
+
+def make_shape(batch, prompt_len, resp_len, n_heads, n_kv_heads, head_dim, softmax_scale=None):
+    s = archer_shape()
+    s.batch, s.prompt_len, s.resp_len = int(batch), int(prompt_len), int(resp_len)
+    s.n_heads, s.n_kv_heads, s.head_dim = int(n_heads), int(n_kv_heads), int(head_dim)
+    s.softmax_scale = float(softmax_scale) if softmax_scale else 0.0
+    return s
+
+
+def _expect(t, shape, what):
+    if tuple(t.shape) != tuple(shape):
+        raise ValueError(f"{what} has shape {tuple(t.shape)}, expected {tuple(shape)}")
+
+
+def archer_attn_step(shape: archer_shape, q_resp, k_cache, v_cache, k_resp, v_resp, out, lse=None,
+                     workspace=None, stream=None):
+    """Cached response step (Sec. 4.1, Eq. archer-attention); see include/archer.h."""
+    B, P, G, Hq, Hkv, D = (shape.batch, shape.prompt_len, shape.resp_len, shape.n_heads, shape.n_kv_heads,
+                           shape.head_dim)
+    bf = torch.bfloat16
+    _expect(q_resp, (B, G, Hq, D), "q_resp")
+    _expect(k_resp, (B, G, Hkv, D), "k_resp")
+    _expect(v_resp, (B, G, Hkv, D), "v_resp")
+    _expect(out, (B, G, Hq, D), "out")
+    if P > 0:
+        _expect(k_cache, (B, P, Hkv, D), "k_cache")
+        _expect(v_cache, (B, P, Hkv, D), "v_cache")
+    if lse is not None:
+        _expect(lse, (B, Hq, G), "lse")
+    ws = workspace
+    _raise(lib.archer_attn_step(ctypes.byref(shape), _ptr(q_resp, bf, "q_resp"), _ptr(k_cache, bf, "k_cache"),
+                                _ptr(v_cache, bf, "v_cache"), _ptr(k_resp, bf, "k_resp"), _ptr(v_resp, bf, "v_resp"),
+                                _ptr(out, bf, "out"), _ptr(lse, torch.float32, "lse"), _ptr(ws, None, "workspace"),
+                                ctypes.c_size_t(0 if ws is None else ws.numel() * ws.element_size()),
+                                _stream(stream)))
+
+
+def archer_prompt_refresh(shape: archer_shape, q_all, k_prompt_new, v_prompt_new, k_resp, v_resp, out,
+                          lse=None, k_cache=None, v_cache=None, refresh_flags=None, workspace=None, stream=None):
+    """Prompt refresh (Sec. 4.2, Algorithm 1's FullForward); see include/archer.h."""
+    B, P, G, Hq, Hkv, D = (shape.batch, shape.prompt_len, shape.resp_len, shape.n_heads, shape.n_kv_heads,
+                           shape.head_dim)
+    N = P + G
+    bf = torch.bfloat16
+    _expect(q_all, (B, N, Hq, D), "q_all")
+    _expect(k_resp, (B, G, Hkv, D), "k_resp")
+    _expect(v_resp, (B, G, Hkv, D), "v_resp")
+    _expect(out, (B, N, Hq, D), "out")
+    if k_cache is None:
+        k_cache = k_prompt_new
+    if v_cache is None:
+        v_cache = v_prompt_new
+    if P > 0:
+        for t, n in ((k_prompt_new, "k_prompt_new"), (v_prompt_new, "v_prompt_new"), (k_cache, "k_cache"),
+                     (v_cache, "v_cache")):
+            _expect(t, (B, P, Hkv, D), n)
+    if lse is not None:
+        _expect(lse, (B, Hq, N), "lse")
+    if refresh_flags is not None:
+        _expect(refresh_flags, (B,), "refresh_flags")
+    ws = workspace
+    _raise(lib.archer_prompt_refresh(
+        ctypes.byref(shape), _ptr(q_all, bf, "q_all"), _ptr(k_prompt_new, bf, "k_prompt_new"),
+        _ptr(v_prompt_new, bf, "v_prompt_new"), _ptr(k_resp, bf, "k_resp"), _ptr(v_resp, bf, "v_resp"),
+        _ptr(out, bf, "out"), _ptr(lse, torch.float32, "lse"), _ptr(k_cache, bf, "k_cache"),
+        _ptr(v_cache, bf, "v_cache"), _ptr(refresh_flags, torch.uint8, "refresh_flags"), _ptr(ws, None, "workspace"),
+        ctypes.c_size_t(0 if ws is None else ws.numel() * ws.element_size()), _stream(stream)))
+
+
+def archer_attn_workspace_size(shape: archer_shape, n_queries: int) -> int:
+    return int(lib.archer_attn_workspace_size(ctypes.byref(shape), int(n_queries)))
+
+
+def archer_decode_scores_workspace_size(rows: int, vocab: int) -> int:
+    return int(lib.archer_decode_scores_workspace_size(int(rows), int(vocab)))
+
+
+_ws_cache: dict = {}
+
+
+def scores_workspace(rows: int, vocab: int, device=None) -> torch.Tensor | None:
+    """A zero-filled workspace for archer_decode_scores, cached per (device, size).
+    Calls that may overlap on the GPU must not share one."""
+    n = archer_decode_scores_workspace_size(rows, vocab)
+    if n == 0:
+        return None
+    dev = torch.device("cuda", torch.cuda.current_device()) if device is None else torch.device(device)
+    key = (dev, n)
+    if key not in _ws_cache:
+        _ws_cache[key] = torch.zeros(n, dtype=torch.uint8, device=dev)
+    return _ws_cache[key]
+
+
+def archer_decode_scores(logits, max_prob, top1, margin, mask_state=None, cur_tokens=None, cur_prob=None,
+                         vocab=None, workspace=None, stream=None):
+    """Decoder scoring; logits [B, G, row_stride] or [rows, row_stride] (bf16 or fp32).
+    Outputs are flat [rows] tensors (fp32, int32, fp32, fp32)."""
+    if logits.dtype == torch.bfloat16:
+        dtype = ARCHER_DTYPE_BF16
+    elif logits.dtype == torch.float32:
+        dtype = ARCHER_DTYPE_F32
+    else:
+        raise TypeError("logits must be bf16 or fp32")
+    if logits.dim() == 3:
+        batch, resp_len, stride = logits.shape
+    elif logits.dim() == 2:
+        batch, (resp_len, stride) = 1, logits.shape
+    else:
+        raise ValueError("logits must be [B, G, V] or [rows, V]")
+    vocab = stride if vocab is None else int(vocab)
+    rows = batch * resp_len
+    for t, n, dt in ((max_prob, "max_prob", torch.float32), (top1, "top1", torch.int32),
+                     (margin, "margin", torch.float32)):
+        if t.numel() != rows or t.dtype != dt:
+            raise ValueError(f"{n} must hold {rows} {dt} values")
+    if cur_prob is not None and (cur_prob.numel() != rows or cur_prob.dtype != torch.float32):
+        raise ValueError("cur_prob must hold rows fp32 values")
+    if workspace is None:
+        workspace = scores_workspace(rows, vocab, logits.device)
+    ws_bytes = 0 if workspace is None else workspace.numel() * workspace.element_size()
+    _raise(lib.archer_decode_scores(
+        batch, resp_len, vocab, dtype, _ptr(logits, None, "logits"), ctypes.c_int64(stride),
+        _ptr(mask_state, torch.uint8, "mask_state"), _ptr(cur_tokens, torch.int32, "cur_tokens"),
+        _ptr(max_prob, None, "max_prob"), _ptr(top1, None, "top1"), _ptr(margin, None, "margin"),
+        _ptr(cur_prob, None, "cur_prob"), _ptr(workspace, None, "workspace"), ctypes.c_size_t(ws_bytes),
+        _stream(stream)))
+
+
+def archer_should_refresh(g_cur, g_anchor, age, K, max_age, update_anchor, dist_out, flag_out, stream=None):
+    """Refresh rule (Sec. 4.2, Eq. archer-distance / archer-controller); see include/archer.h."""
+    B, G = g_cur.shape
+    _expect(g_anchor, (B, G), "g_anchor")
+    _expect(age, (B,), "age")
+    _expect(flag_out, (B,), "flag_out")
+    if dist_out is not None:
+        _expect(dist_out, (B,), "dist_out")
+    i32 = torch.int32
+    _raise(lib.archer_should_refresh(B, G, _ptr(g_cur, i32, "g_cur"), _ptr(g_anchor, i32, "g_anchor"),
+                                     _ptr(age, i32, "age"), int(min(K, K_INFINITE)), int(max_age),
+                                     int(bool(update_anchor)), _ptr(dist_out, i32, "dist_out"),
+                                     _ptr(flag_out, torch.uint8, "flag_out"), _stream(stream)))
+
+
+def archer_cache_rewrite(shape: archer_shape, k_src, v_src, k_dst, v_dst, refresh_flags=None, stream=None):
+    bf = torch.bfloat16
+    _raise(lib.archer_cache_rewrite(ctypes.byref(shape), _ptr(k_src, bf, "k_src"), _ptr(v_src, bf, "v_src"),
+                                    _ptr(k_dst, bf, "k_dst"), _ptr(v_dst, bf, "v_dst"),
+                                    _ptr(refresh_flags, torch.uint8, "refresh_flags"), _stream(stream)))
+
+
+def archer_check_device(stream=None):
+    _raise(lib.archer_check_device(_stream(stream)))
+
+
+def archer_version() -> int:
+    return int(lib.archer_version())
+
+
+def default_scale(head_dim: int) -> float:
+    return 1.0 / math.sqrt(head_dim)

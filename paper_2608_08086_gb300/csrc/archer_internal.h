@@ -1,0 +1,57 @@
+// Host-side declarations shared by the C-ABI layer (api.cu) and the kernel
+// translation units.  Not part of the public interface (include/archer.h).
+#pragma once
+
+#include <cuda_runtime.h>
+
+#include <cstddef>
+#include <cstdint>
+
+#include "../../include/archer.h"
+
+namespace archer {
+
+// Records a formatted message as this thread's archer_last_error().
+void set_error(const char* fmt, ...);
+
+// Maps a CUDA error to ARCHER_ERR_CUDA with a message naming `what`.
+int cuda_status(cudaError_t e, const char* what);
+
+// Device error word (kernels OR kErr* bits into it).
+int* device_error_word();
+
+struct AttnCall {
+  int B, P, G, Hq, Hkv, D;
+  float scale;            // > 0
+  const void* q;          // [B, M, Hq, D]
+  int M;                  // rows of q / out
+  const void* kp_refresh; // prompt K/V used by refreshed sequences
+  const void* vp_refresh;
+  const void* kp_cached;  // prompt K/V used by sequences taking the cached step
+  const void* vp_cached;
+  const void* kg;
+  const void* vg;
+  void* out;
+  float* lse;
+  const uint8_t* flags;   // nullable
+  int default_refresh;    // used when flags == nullptr
+  int q_begin_refresh;    // first query row of a refreshed sequence
+  int q_begin_cached;     // first query row of a cached sequence
+};
+
+int attn_launch(const AttnCall& c, cudaStream_t stream);
+
+int cache_rewrite_launch(int B, size_t bytes_per_seq, const void* k_src, const void* v_src,
+                         void* k_dst, void* v_dst, const uint8_t* flags, cudaStream_t stream);
+
+int decode_scores_launch(int rows, int vocab, int dtype, const void* logits, int64_t row_stride,
+                         const uint8_t* mask_state, const int32_t* cur_tokens, float* max_prob,
+                         int32_t* top1, float* margin, float* cur_prob, void* workspace,
+                         size_t ws_bytes, cudaStream_t stream);
+size_t decode_scores_ws_bytes(int rows, int vocab);
+
+int should_refresh_launch(int B, int G, const int32_t* g_cur, int32_t* g_anchor, int32_t* age,
+                          int K, int max_age, int update_anchor, int32_t* dist, uint8_t* flag,
+                          cudaStream_t stream);
+
+}  // namespace archer

@@ -1,0 +1,341 @@
+// Decoder scoring for sm_103a: per row of vocabulary logits, the fp32
+// softmax's max probability, the top-1 id (lowest index on ties), the
+// top-1/top-2 probability margin and optionally p(current token).  These are
+// the inputs of the rollback decoder's confidence rule (Sec. 6; the decision
+// margin of Eq. theory-margin is taken on them).
+//
+// HBM-streaming reduction, one pass over the logits:
+//   * a row is cut into chunks of kThreads * kUnroll 16-byte words; one CTA
+//     per (row, chunk) issues all its loads up front (coalesced, 16 B/thread);
+//   * pass A over the registers: max and second value per thread (for bf16
+//     with packed bf16x2 max/min, 1.5 ops per element), CTA-reduced;
+//   * pass B: sum of 2^((z - m) log2 e) with the CTA max m -- exactly one ex2
+//     per element; the lowest index of m is found by the threads holding it;
+//   * chunk partials (m, sum, top-2 value, index) go to the workspace; the
+//     last CTA of a row (ticket counter) merges them and writes the outputs
+//     and re-zeroes the counter.  A row of one chunk skips the workspace.
+
+#include <cfloat>
+#include <cmath>
+
+#include "archer_device.cuh"
+#include "archer_internal.h"
+
+namespace archer {
+namespace {
+
+constexpr int kThreads = 256;
+constexpr int kUnroll = 8;                       // 16-byte words per thread per chunk
+constexpr int kWordsPerChunk = kThreads * kUnroll;
+constexpr float kLog2e = 1.4426950408889634f;
+
+struct Partial {
+  float m;      // chunk max
+  float s;      // sum of 2^((z - m) log2 e) over the chunk
+  float t2;     // chunk second value (multiset: equals m on a tie)
+  int idx;      // lowest index attaining m
+};
+
+// Merge of (top1, top2) value pairs with multiset semantics.
+__device__ __forceinline__ void merge_top2(float& a1, float& a2, float b1, float b2) {
+  const float hi = fmaxf(a1, b1);
+  const float lo = fminf(a1, b1);
+  a2 = fmaxf(lo, fmaxf(a2, b2));
+  a1 = hi;
+}
+
+template <typename T>
+struct Vec;
+template <>
+struct Vec<__nv_bfloat16> {
+  static constexpr int kElems = 8;
+};
+template <>
+struct Vec<float> {
+  static constexpr int kElems = 4;
+};
+
+__device__ __forceinline__ void unpack(const uint4& w, float (&v)[8], __nv_bfloat16*) {
+  const uint32_t u[4] = {w.x, w.y, w.z, w.w};
+#pragma unroll
+  for (int i = 0; i < 4; ++i) {
+    v[2 * i] = __uint_as_float(u[i] << 16);
+    v[2 * i + 1] = __uint_as_float(u[i] & 0xFFFF0000u);
+  }
+}
+__device__ __forceinline__ void unpack(const uint4& w, float (&v)[4], float*) {
+  v[0] = __uint_as_float(w.x);
+  v[1] = __uint_as_float(w.y);
+  v[2] = __uint_as_float(w.z);
+  v[3] = __uint_as_float(w.w);
+}
+
+// Block-wide reduction of (top1, top2) and, second, of (sum, min index).
+struct Smem {
+  float a[kThreads / 32];
+  float b[kThreads / 32];
+  int i[kThreads / 32];
+  float m_block, t2_block;
+  int last;
+};
+
+__device__ __forceinline__ void block_top2(float& t1, float& t2, Smem& sm) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    const float b1 = __shfl_xor_sync(0xffffffffu, t1, o);
+    const float b2 = __shfl_xor_sync(0xffffffffu, t2, o);
+    merge_top2(t1, t2, b1, b2);
+  }
+  const int w = threadIdx.x >> 5, l = threadIdx.x & 31;
+  if (l == 0) { sm.a[w] = t1; sm.b[w] = t2; }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    float x1 = sm.a[0], x2 = sm.b[0];
+    for (int k = 1; k < kThreads / 32; ++k) merge_top2(x1, x2, sm.a[k], sm.b[k]);
+    sm.m_block = x1;
+    sm.t2_block = x2;
+  }
+  __syncthreads();
+  t1 = sm.m_block;
+  t2 = sm.t2_block;
+}
+
+__device__ __forceinline__ void block_sum_minidx(float& s, int& idx, Smem& sm) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    s += __shfl_xor_sync(0xffffffffu, s, o);
+    idx = min(idx, __shfl_xor_sync(0xffffffffu, idx, o));
+  }
+  const int w = threadIdx.x >> 5, l = threadIdx.x & 31;
+  __syncthreads();   // sm.a reused
+  if (l == 0) { sm.a[w] = s; sm.i[w] = idx; }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    float ss = 0.f;
+    int ii = INT_MAX;
+    for (int k = 0; k < kThreads / 32; ++k) { ss += sm.a[k]; ii = min(ii, sm.i[k]); }
+    s = ss;
+    idx = ii;
+  }
+}
+
+__device__ __forceinline__ float load_logit(const void* row, int dtype, int j) {
+  return dtype == ARCHER_DTYPE_BF16
+             ? __bfloat162float(static_cast<const __nv_bfloat16*>(row)[j])
+             : static_cast<const float*>(row)[j];
+}
+
+// Writes the outputs of one row from its merged (M, S, top2, idx).
+__device__ __forceinline__ void write_row(int row, float M, float S, float t2, int idx, const void* zrow,
+                                          int dtype, int vocab, const uint8_t* mask_state,
+                                          const int32_t* cur_tokens, float* max_prob, int32_t* top1,
+                                          float* margin, float* cur_prob) {
+  const float inv = 1.0f / S;
+  max_prob[row] = inv;
+  top1[row] = idx;
+  margin[row] = vocab > 1 ? (1.0f - ex2_approx((t2 - M) * kLog2e)) * inv : inv;
+  if (cur_prob) {
+    float c = 0.f;
+    const bool masked = mask_state && mask_state[row] != 0;
+    if (cur_tokens && !masked) {
+      const int t = cur_tokens[row];
+      if (t >= 0 && t < vocab) c = ex2_approx((load_logit(zrow, dtype, t) - M) * kLog2e) * inv;
+    }
+    cur_prob[row] = c;
+  }
+}
+
+template <typename T>
+__global__ void __launch_bounds__(kThreads)
+decode_scores_kernel(const T* __restrict__ logits, int64_t row_stride, int vocab, int chunks,
+                     const uint8_t* __restrict__ mask_state, const int32_t* __restrict__ cur_tokens,
+                     float* __restrict__ max_prob, int32_t* __restrict__ top1, float* __restrict__ margin,
+                     float* __restrict__ cur_prob, int* __restrict__ counters, Partial* __restrict__ parts) {
+  constexpr int E = Vec<T>::kElems;              // elements per 16-byte word
+  constexpr int dtype = sizeof(T) == 2 ? ARCHER_DTYPE_BF16 : ARCHER_DTYPE_F32;
+  __shared__ Smem sm;
+  const int row = blockIdx.x / chunks;
+  const int chunk = blockIdx.x - row * chunks;
+  const T* zrow = logits + row * row_stride;
+  const int64_t chunk_elem0 = static_cast<int64_t>(chunk) * kWordsPerChunk * E;
+
+  // ---- issue all loads (word u of this thread covers elements e0 .. e0+E-1)
+  uint4 w[kUnroll];
+  const uint4* zw = reinterpret_cast<const uint4*>(zrow);
+#pragma unroll
+  for (int u = 0; u < kUnroll; ++u) {
+    const int64_t e0 = chunk_elem0 + (static_cast<int64_t>(u) * kThreads + threadIdx.x) * E;
+    if (e0 + E <= vocab) {
+      w[u] = __ldcs(zw + e0 / E);                 // streamed once: evict-first
+    } else {
+      // ragged tail: element-wise, -inf past the vocabulary
+      float v[E];
+#pragma unroll
+      for (int e = 0; e < E; ++e) v[e] = (e0 + e < vocab) ? load_logit(zrow, dtype, (int)(e0 + e)) : -INFINITY;
+      if constexpr (E == 8) {   // exact: every value is a bf16 value or -inf
+        w[u] = make_uint4(pack_bf16x2(v[0], v[1]), pack_bf16x2(v[2], v[3]), pack_bf16x2(v[4], v[5]),
+                          pack_bf16x2(v[6], v[7]));
+      } else {
+        w[u] = make_uint4(__float_as_uint(v[0]), __float_as_uint(v[1]), __float_as_uint(v[2]),
+                          __float_as_uint(v[3]));
+      }
+    }
+  }
+
+  // ---- pass A: per-thread top-2 values, then CTA-wide
+  float t1 = -INFINITY, t2 = -INFINITY;
+  if constexpr (E == 8) {
+    __nv_bfloat162 M1 = __floats2bfloat162_rn(-INFINITY, -INFINITY);
+    __nv_bfloat162 M2 = M1;
+#pragma unroll
+    for (int u = 0; u < kUnroll; ++u) {
+      const uint32_t q[4] = {w[u].x, w[u].y, w[u].z, w[u].w};
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        const __nv_bfloat162 x = *reinterpret_cast<const __nv_bfloat162*>(&q[i]);
+        M2 = __hmax2(M2, __hmin2(M1, x));
+        M1 = __hmax2(M1, x);
+      }
+    }
+    const float a = __low2float(M1), c = __high2float(M1);
+    t1 = fmaxf(a, c);
+    t2 = fmaxf(fminf(a, c), fmaxf(__low2float(M2), __high2float(M2)));
+  } else {
+#pragma unroll
+    for (int u = 0; u < kUnroll; ++u) {
+      float v[4];
+      unpack(w[u], v, (float*)nullptr);
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        t2 = fmaxf(t2, fminf(t1, v[e]));
+        t1 = fmaxf(t1, v[e]);
+      }
+    }
+  }
+  const float my_t1 = t1;
+  float m_blk = t1, t2_blk = t2;
+  block_top2(m_blk, t2_blk, sm);
+
+  // ---- pass B: sum of exps relative to the CTA max; lowest index of the max
+  // A chunk whose logits are all -inf contributes a zero sum (not NaN).
+  const float neg_m = (m_blk == -INFINITY) ? 0.f : -m_blk * kLog2e;
+  float s = 0.f;
+#pragma unroll
+  for (int u = 0; u < kUnroll; ++u) {
+    float v[E];
+    unpack(w[u], v, (T*)nullptr);
+#pragma unroll
+    for (int e = 0; e < E; ++e) s += ex2_approx(fmaf(v[e], kLog2e, neg_m));
+  }
+  int idx = INT_MAX;
+  if (my_t1 == m_blk) {
+    for (int u = 0; u < kUnroll && idx == INT_MAX; ++u) {
+      float v[E];
+      unpack(w[u], v, (T*)nullptr);
+      const int64_t e0 = chunk_elem0 + (static_cast<int64_t>(u) * kThreads + threadIdx.x) * E;
+#pragma unroll
+      for (int e = E - 1; e >= 0; --e)
+        if (v[e] == m_blk) idx = (int)(e0 + e);
+    }
+  }
+  block_sum_minidx(s, idx, sm);
+
+  if (chunks == 1) {
+    if (threadIdx.x == 0)
+      write_row(row, m_blk, s, t2_blk, idx, zrow, dtype, vocab, mask_state, cur_tokens, max_prob, top1, margin,
+                cur_prob);
+    return;
+  }
+
+  // ---- publish the chunk partial; the last CTA of the row merges
+  if (threadIdx.x == 0) {
+    Partial pt;
+    pt.m = m_blk; pt.s = s; pt.t2 = t2_blk; pt.idx = idx;
+    parts[static_cast<size_t>(row) * chunks + chunk] = pt;
+    __threadfence();
+    const int ticket = atomicAdd(&counters[row], 1);
+    sm.last = (ticket == chunks - 1);
+  }
+  __syncthreads();
+  if (!sm.last) return;
+  __threadfence();
+  if (threadIdx.x < 32) {
+    // warp 0 merges the chunk partials of this row
+    float M = -INFINITY, T2 = -INFINITY;
+    const volatile Partial* vp = parts + static_cast<size_t>(row) * chunks;
+    for (int c = threadIdx.x; c < chunks; c += 32) merge_top2(M, T2, vp[c].m, vp[c].t2);
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      const float b1 = __shfl_xor_sync(0xffffffffu, M, o);
+      const float b2 = __shfl_xor_sync(0xffffffffu, T2, o);
+      merge_top2(M, T2, b1, b2);
+    }
+    float S = 0.f;
+    int I = INT_MAX;
+    for (int c = threadIdx.x; c < chunks; c += 32) {
+      const float mc = vp[c].m;
+      S += vp[c].s * ex2_approx((mc - M) * kLog2e);
+      if (mc == M) I = min(I, (int)vp[c].idx);
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+      S += __shfl_xor_sync(0xffffffffu, S, o);
+      I = min(I, __shfl_xor_sync(0xffffffffu, I, o));
+    }
+    if (threadIdx.x == 0) {
+      write_row(row, M, S, T2, I, zrow, dtype, vocab, mask_state, cur_tokens, max_prob, top1, margin, cur_prob);
+      counters[row] = 0;   // leave the workspace zero-filled for the next call
+    }
+  }
+}
+
+int chunks_for(int vocab, int dtype) {
+  const int per_chunk = kWordsPerChunk * (dtype == ARCHER_DTYPE_BF16 ? 8 : 4);
+  return (vocab + per_chunk - 1) / per_chunk;
+}
+
+}  // namespace
+
+size_t decode_scores_ws_bytes(int rows, int vocab) {
+  // Sized for fp32 logits, which need twice the chunks of bf16 for one vocabulary.
+  const int chunks = chunks_for(vocab, ARCHER_DTYPE_F32);
+  if (chunks <= 1 || rows <= 0) return 0;
+  const size_t counters = ((static_cast<size_t>(rows) * sizeof(int) + 255) / 256) * 256;
+  return counters + static_cast<size_t>(rows) * chunks * sizeof(Partial);
+}
+
+int decode_scores_launch(int rows, int vocab, int dtype, const void* logits, int64_t row_stride,
+                         const uint8_t* mask_state, const int32_t* cur_tokens, float* max_prob, int32_t* top1,
+                         float* margin, float* cur_prob, void* workspace, size_t ws_bytes, cudaStream_t stream) {
+  if (rows == 0) return ARCHER_OK;
+  const int chunks = chunks_for(vocab, dtype);
+  int* counters = nullptr;
+  Partial* parts = nullptr;
+  if (chunks > 1) {
+    const size_t need = decode_scores_ws_bytes(rows, vocab);
+    if (workspace == nullptr || ws_bytes < need) {
+      set_error("decode_scores needs a zero-filled workspace of %zu bytes (got %zu)", need, ws_bytes);
+      return ARCHER_ERR_ARG;
+    }
+    counters = static_cast<int*>(workspace);
+    parts = reinterpret_cast<Partial*>(static_cast<char*>(workspace) +
+                                       ((static_cast<size_t>(rows) * sizeof(int) + 255) / 256) * 256);
+  }
+  const long long grid = static_cast<long long>(rows) * chunks;
+  if (grid > 0x7FFFFFFFll) {
+    set_error("decode_scores grid too large");
+    return ARCHER_ERR_UNSUPPORTED;
+  }
+  if (dtype == ARCHER_DTYPE_BF16) {
+    decode_scores_kernel<__nv_bfloat16><<<(unsigned)grid, kThreads, 0, stream>>>(
+        static_cast<const __nv_bfloat16*>(logits), row_stride, vocab, chunks, mask_state, cur_tokens, max_prob, top1,
+        margin, cur_prob, counters, parts);
+  } else {
+    decode_scores_kernel<float><<<(unsigned)grid, kThreads, 0, stream>>>(
+        static_cast<const float*>(logits), row_stride, vocab, chunks, mask_state, cur_tokens, max_prob, top1, margin,
+        cur_prob, counters, parts);
+  }
+  return cuda_status(cudaGetLastError(), "decode_scores launch");
+}
+
+}  // namespace archer

@@ -1,0 +1,84 @@
+"""The C-ABI library builds, loads, exports every declared symbol and rejects
+bad arguments before touching the device (no GPU needed)."""
+import ctypes
+import os
+import re
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    from paper_2608_08086_gb300 import build
+    return ctypes.CDLL(build.build())
+
+
+def declared_functions():
+    names = []
+    for fn in os.listdir(os.path.join(ROOT, "include")):
+        if fn.endswith(".h"):
+            text = open(os.path.join(ROOT, "include", fn)).read()
+            text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+            names += re.findall(r"\b(archer_[a-z0-9_]+)\s*\(", text)
+    return sorted(set(names))
+
+
+def test_every_declared_symbol_is_exported(lib):
+    names = declared_functions()
+    assert len(names) >= 10
+    missing = [n for n in names if not hasattr(lib, n)]
+    assert not missing, f"declared but not exported: {missing}"
+
+
+def test_status_strings_and_version(lib):
+    lib.archer_status_string.restype = ctypes.c_char_p
+    assert lib.archer_status_string(0) == b"ok"
+    assert lib.archer_status_string(-4) == b"device wait timed out"
+    assert lib.archer_version() >= 100
+
+
+class Shape(ctypes.Structure):
+    _fields_ = [("batch", ctypes.c_int), ("prompt_len", ctypes.c_int), ("resp_len", ctypes.c_int),
+                ("n_heads", ctypes.c_int), ("n_kv_heads", ctypes.c_int), ("head_dim", ctypes.c_int),
+                ("softmax_scale", ctypes.c_float)]
+
+
+def _attn_step(lib, shape, ptr=0x10000):
+    f = lib.archer_attn_step
+    f.argtypes = [ctypes.POINTER(Shape)] + [ctypes.c_void_p] * 8 + [ctypes.c_size_t, ctypes.c_void_p]
+    f.restype = ctypes.c_int
+    p = ctypes.c_void_p(ptr)
+    return f(ctypes.byref(shape), p, p, p, p, p, p, None, None, 0, None)
+
+
+def test_bad_shapes_rejected_before_any_launch(lib):
+    lib.archer_last_error.restype = ctypes.c_char_p
+    assert _attn_step(lib, Shape(1, 4, 4, 3, 2, 128, 0.0)) == -1          # Hq % Hkv != 0
+    assert b"multiple" in lib.archer_last_error()
+    assert _attn_step(lib, Shape(1, 4, 0, 2, 2, 128, 0.0)) == -1          # G = 0
+    assert _attn_step(lib, Shape(1, 4, 4, 2, 2, 96, 0.0)) == -2           # D unsupported
+    assert _attn_step(lib, Shape(1, 4, 4, 2, 2, 128, float("nan"))) == -1
+    assert _attn_step(lib, Shape(1, 4, 4, 2, 2, 128, 0.0), ptr=0x10008) == -1   # misaligned
+    assert b"aligned" in lib.archer_last_error()
+    f = lib.archer_attn_step
+    s = Shape(1, 4, 4, 2, 2, 128, 0.0)
+    assert f(ctypes.byref(s), None, None, None, None, None, None, None, None, 0, None) == -1
+    assert _attn_step(lib, Shape(0, 4, 4, 2, 2, 128, 0.0)) == 0            # empty batch: no-op
+
+
+def test_bad_scoring_and_rule_arguments_rejected(lib):
+    f = lib.archer_decode_scores
+    f.argtypes = [ctypes.c_int] * 4 + [ctypes.c_void_p, ctypes.c_int64] + [ctypes.c_void_p] * 7 + [
+        ctypes.c_size_t, ctypes.c_void_p]
+    p = ctypes.c_void_p(0x10000)
+    assert f(1, 4, 100, 0, p, 50, None, None, p, p, p, None, None, 0, None) == -1     # stride < vocab
+    assert f(1, 4, 100, 0, p, 100, None, None, p, p, p, None, None, 0, None) == -1    # 200 B stride
+    assert f(1, 4, 104, 7, p, 104, None, None, p, p, p, None, None, 0, None) == -2    # dtype
+    assert f(1, 4, 104, 0, p, 104, None, None, None, p, p, None, None, 0, None) == -1  # null output
+    g = lib.archer_should_refresh
+    g.argtypes = [ctypes.c_int, ctypes.c_int] + [ctypes.c_void_p] * 3 + [ctypes.c_int] * 3 + [ctypes.c_void_p] * 3
+    assert g(-1, 4, p, p, p, 1, 0, 1, p, p, None) == -1
+    assert g(2, 4, None, p, p, 1, 0, 1, p, p, None) == -1
+    assert g(0, 4, None, None, None, 1, 0, 1, None, None, None) == 0

@@ -1,0 +1,319 @@
+"""GPU-vs-oracle parity of every hot-path call, through the C ABI.
+
+Acceptance (stated up front and used everywhere below):
+  * attention output:  |gpu - ref| <= 2e-2 + 2e-2 |ref|   (bf16 inputs, fp32 accumulation)
+  * attention lse:     |gpu - ref| <= 1e-3 + 1e-3 |ref|
+  * refresh flags, distances, anchors, ages, cache rewrite: bit-exact
+  * top-1 ids: exact, except rows whose oracle top-1/top-2 probability margin < 1e-4
+  * max_prob, margin, cur_prob: |gpu - ref| <= 1e-5 + 1e-4 |ref|
+"""
+import math
+
+import numpy as np
+import pytest
+import torch
+
+from oracle import oracle as O
+from paper_2608_08086_gb300 import synth
+
+pytestmark = pytest.mark.gpu
+
+ATOL = RTOL = 2e-2
+LSE_TOL = 1e-3
+P_ATOL, P_RTOL = 1e-5, 1e-4
+MARGIN_EXCLUDE = 1e-4
+
+
+@pytest.fixture(scope="module")
+def A():
+    if not torch.cuda.is_available():
+        pytest.fail("the gpu tests need a CUDA device")
+    from paper_2608_08086_gb300 import archer
+    return archer
+
+
+def dev_bf16(bits):
+    return torch.from_numpy(np.ascontiguousarray(bits).view(np.int16)).view(torch.bfloat16).cuda()
+
+
+def host_f64(t):
+    if t.dtype == torch.bfloat16:
+        return synth.bf16_bits_to_f64(t.contiguous().view(torch.int16).cpu().numpy().view(np.uint16))
+    return t.double().cpu().numpy()
+
+
+def assert_attn_close(got, ref, what):
+    err = np.abs(got - ref)
+    bound = ATOL + RTOL * np.abs(ref)
+    bad = err > bound
+    assert not bad.any(), (f"{what}: {bad.sum()} of {bad.size} elements out of tolerance; "
+                           f"max err {err.max():.3e} at {np.unravel_index(np.argmax(err - bound), err.shape)}")
+
+
+def assert_lse_close(got, ref, what):
+    err = np.abs(got - ref)
+    assert (err <= LSE_TOL + LSE_TOL * np.abs(ref)).all(), f"{what}: lse max err {err.max():.3e}"
+
+
+ATTN_CASES = [
+    # B, P, G, Hq, Hkv, D
+    (1, 128, 64, 4, 4, 64),        # the tiny workload
+    (2, 100, 37, 8, 2, 128),       # ragged prompt and response tiles, GQA 4:1
+    (1, 0, 200, 2, 1, 128),        # P = 0: response-only attention
+    (1, 300, 1, 4, 4, 64),         # G = 1
+    (2, 256, 256, 2, 2, 128),      # several full tiles in both segments
+    (1, 129, 130, 4, 1, 64),       # one-past-a-tile in both segments, GQA 4:1
+    (1, 640, 384, 7, 1, 128),      # GQA 7:1, 8 KV tiles
+]
+
+
+def _inputs(case, seed, std=None):
+    B, P, G, Hq, Hkv, D = case
+    sh = synth.AttnShape(B, P, G, Hq, Hkv, D)
+    bits = synth.attn_inputs(sh, seed=seed, std=std)
+    return sh, bits, {k: synth.bf16_bits_to_f64(v) for k, v in bits.items()}
+
+
+@pytest.mark.parametrize("case", ATTN_CASES)
+@pytest.mark.parametrize("sharp", [False, True])
+def test_attn_step_matches_oracle(A, case, sharp):
+    B, P, G, Hq, Hkv, D = case
+    sh, bits, x = _inputs(case, seed=21, std=1.0 if sharp else None)
+    scale = 1.0 if sharp else 1.0 / math.sqrt(D)
+    d = {k: dev_bf16(v) for k, v in bits.items()}
+    q_resp = d["q_all"][:, P:].contiguous()
+    out = torch.empty(B, G, Hq, D, dtype=torch.bfloat16, device="cuda")
+    lse = torch.empty(B, Hq, G, dtype=torch.float32, device="cuda")
+    A.archer_attn_step(A.make_shape(B, P, G, Hq, Hkv, D, scale), q_resp, d["k_cache"], d["v_cache"],
+                       d["k_resp"], d["v_resp"], out, lse)
+    torch.cuda.synchronize()
+    A.archer_check_device()
+    ref, ref_lse = O.attn_step(x["q_all"][:, P:], x["k_cache"], x["v_cache"], x["k_resp"], x["v_resp"], scale)
+    assert_attn_close(host_f64(out), ref, f"step {case} sharp={sharp}")
+    assert_lse_close(host_f64(lse), ref_lse, f"step {case}")
+
+
+@pytest.mark.parametrize("case", ATTN_CASES)
+def test_prompt_refresh_matches_oracle(A, case):
+    B, P, G, Hq, Hkv, D = case
+    sh, bits, x = _inputs(case, seed=22)
+    scale = 1.0 / math.sqrt(D)
+    d = {k: dev_bf16(v) for k, v in bits.items()}
+    N = P + G
+    out = torch.empty(B, N, Hq, D, dtype=torch.bfloat16, device="cuda")
+    lse = torch.empty(B, Hq, N, dtype=torch.float32, device="cuda")
+    kc, vc = d["k_cache"].clone(), d["v_cache"].clone()
+    A.archer_prompt_refresh(A.make_shape(B, P, G, Hq, Hkv, D), d["q_all"], d["k_prompt"], d["v_prompt"],
+                            d["k_resp"], d["v_resp"], out, lse, kc, vc)
+    torch.cuda.synchronize()
+    A.archer_check_device()
+    ref, ref_lse, rkc, rvc = O.prompt_refresh(x["q_all"], x["k_prompt"], x["v_prompt"], x["k_resp"], x["v_resp"],
+                                              x["k_cache"], x["v_cache"], scale)
+    assert_attn_close(host_f64(out), ref, f"refresh {case}")
+    assert_lse_close(host_f64(lse), ref_lse, f"refresh {case}")
+    if P > 0:
+        assert torch.equal(kc, d["k_prompt"]) and torch.equal(vc, d["v_prompt"])
+
+
+def test_prompt_refresh_mixed_flags(A):
+    B, P, G, Hq, Hkv, D = 3, 200, 100, 4, 2, 128
+    sh, bits, x = _inputs((B, P, G, Hq, Hkv, D), seed=23)
+    scale = 1.0 / math.sqrt(D)
+    d = {k: dev_bf16(v) for k, v in bits.items()}
+    flags = np.array([0, 1, 0], dtype=np.uint8)
+    N = P + G
+    sentinel = 3.0
+    out = torch.full((B, N, Hq, D), sentinel, dtype=torch.bfloat16, device="cuda")
+    lse = torch.full((B, Hq, N), sentinel, dtype=torch.float32, device="cuda")
+    kc, vc = d["k_cache"].clone(), d["v_cache"].clone()
+    A.archer_prompt_refresh(A.make_shape(B, P, G, Hq, Hkv, D), d["q_all"], d["k_prompt"], d["v_prompt"],
+                            d["k_resp"], d["v_resp"], out, lse, kc, vc,
+                            refresh_flags=torch.from_numpy(flags).cuda())
+    torch.cuda.synchronize()
+    ref, ref_lse, rkc, rvc = O.prompt_refresh(x["q_all"], x["k_prompt"], x["v_prompt"], x["k_resp"], x["v_resp"],
+                                              x["k_cache"], x["v_cache"], scale, flags=flags,
+                                              out=np.full((B, N, Hq, D), sentinel),
+                                              lse=np.full((B, Hq, N), sentinel))
+    assert_attn_close(host_f64(out), ref, "mixed refresh")
+    assert_lse_close(host_f64(lse), ref_lse, "mixed refresh")
+    np.testing.assert_array_equal(host_f64(kc), rkc)
+    np.testing.assert_array_equal(host_f64(vc), rvc)
+
+
+def test_refresh_every_step_equals_eager_on_gpu(A):
+    # Eq. archer-controller: with the cache just rebuilt, the cached step equals
+    # the refresh pass's response rows.  Same kernel, same tiles: bit-identical.
+    B, P, G, Hq, Hkv, D = 2, 384, 256, 4, 4, 128
+    sh, bits, x = _inputs((B, P, G, Hq, Hkv, D), seed=24)
+    d = {k: dev_bf16(v) for k, v in bits.items()}
+    N = P + G
+    shape = A.make_shape(B, P, G, Hq, Hkv, D)
+    out_full = torch.empty(B, N, Hq, D, dtype=torch.bfloat16, device="cuda")
+    kc, vc = d["k_cache"].clone(), d["v_cache"].clone()
+    A.archer_prompt_refresh(shape, d["q_all"], d["k_prompt"], d["v_prompt"], d["k_resp"], d["v_resp"], out_full,
+                            None, kc, vc)
+    out_step = torch.empty(B, G, Hq, D, dtype=torch.bfloat16, device="cuda")
+    A.archer_attn_step(shape, d["q_all"][:, P:].contiguous(), kc, vc, d["k_resp"], d["v_resp"], out_step)
+    torch.cuda.synchronize()
+    ref = O.attn_step(x["q_all"][:, P:], x["k_prompt"], x["v_prompt"], x["k_resp"], x["v_resp"],
+                      1 / math.sqrt(D))[0]
+    assert_attn_close(host_f64(out_step), ref, "step after refresh")
+    # Tiles of the step start at query row P, those of the refresh pass at 0; with
+    # P a multiple of 128 they coincide and the results are bit-identical.
+    assert torch.equal(out_step, out_full[:, P:])
+
+
+def test_attention_full_size_gqa_long_sampled(A):
+    # Long-prompt GQA workload at full size (B16, 28/4 heads, D128, P4096, G512),
+    # both passes in the launch configuration the bench times; oracle on
+    # sampled rows (rows 0, G-1 and a spread in between; refresh adds P-1, P).
+    B, P, G, Hq, Hkv, D = 16, 4096, 512, 28, 4, 128
+    sh = synth.AttnShape(B, P, G, Hq, Hkv, D)
+    d = synth.device_attn_inputs(sh, "cuda", seed=3)
+    N = P + G
+    scale = 1.0 / math.sqrt(D)
+    shape = A.make_shape(B, P, G, Hq, Hkv, D)
+    out_s = torch.empty(B, G, Hq, D, dtype=torch.bfloat16, device="cuda")
+    q_resp = d["q_all"][:, P:].contiguous()
+    A.archer_attn_step(shape, q_resp, d["k_cache"], d["v_cache"], d["k_resp"], d["v_resp"], out_s)
+    out_r = torch.empty(B, N, Hq, D, dtype=torch.bfloat16, device="cuda")
+    kc, vc = d["k_cache"].clone(), d["v_cache"].clone()
+    A.archer_prompt_refresh(shape, d["q_all"], d["k_prompt"], d["v_prompt"], d["k_resp"], d["v_resp"], out_r,
+                            None, kc, vc)
+    torch.cuda.synchronize()
+    A.archer_check_device()
+    rng = np.random.default_rng(0)
+    for b, h in [(0, 0), (7, 13), (15, 27)]:
+        kvh = h // (Hq // Hkv)
+        kg, vg = host_f64(d["k_resp"][b:b + 1, :, kvh:kvh + 1]), host_f64(d["v_resp"][b:b + 1, :, kvh:kvh + 1])
+        rows_s = np.unique(np.concatenate([[0, G - 1], rng.integers(0, G, 30)]))
+        q = host_f64(q_resp[b:b + 1, rows_s, h:h + 1])
+        kc0, vc0 = host_f64(d["k_cache"][b:b + 1, :, kvh:kvh + 1]), host_f64(d["v_cache"][b:b + 1, :, kvh:kvh + 1])
+        ref, _ = O.attention(q, kc0, vc0, kg, vg, scale)
+        assert_attn_close(host_f64(out_s[b:b + 1, rows_s, h:h + 1]), ref, f"gqa step b{b} h{h}")
+        rows_r = np.unique(np.concatenate([[0, P - 1, P, N - 1], rng.integers(0, N, 30)]))
+        q = host_f64(d["q_all"][b:b + 1, rows_r, h:h + 1])
+        kp, vp = host_f64(d["k_prompt"][b:b + 1, :, kvh:kvh + 1]), host_f64(d["v_prompt"][b:b + 1, :, kvh:kvh + 1])
+        ref, _ = O.attention(q, kp, vp, kg, vg, scale)
+        assert_attn_close(host_f64(out_r[b:b + 1, rows_r, h:h + 1]), ref, f"gqa refresh b{b} h{h}")
+    assert torch.equal(kc, d["k_prompt"]) and torch.equal(vc, d["v_prompt"])
+
+
+# ----------------------------------------------------------------------------
+# decoder scoring
+# ----------------------------------------------------------------------------
+
+def _run_scores(A, z_dev, vocab, mask=None, cur=None):
+    rows = z_dev.shape[0]
+    mp = torch.empty(rows, dtype=torch.float32, device="cuda")
+    t1 = torch.empty(rows, dtype=torch.int32, device="cuda")
+    mg = torch.empty(rows, dtype=torch.float32, device="cuda")
+    cp = torch.empty(rows, dtype=torch.float32, device="cuda") if cur is not None else None
+    A.archer_decode_scores(z_dev, mp, t1, mg, mask_state=mask, cur_tokens=cur, cur_prob=cp, vocab=vocab)
+    torch.cuda.synchronize()
+    res = {"max_prob": mp.cpu().numpy().astype(np.float64), "top1": t1.cpu().numpy(),
+           "margin": mg.cpu().numpy().astype(np.float64)}
+    if cp is not None:
+        res["cur_prob"] = cp.cpu().numpy().astype(np.float64)
+    return res
+
+
+def assert_scores_close(got, ref, what, rows=None):
+    sel = slice(None) if rows is None else rows
+    keep = ref["margin"] >= MARGIN_EXCLUDE
+    mism = (got["top1"] != ref["top1"][sel]) & keep
+    assert not mism.any(), f"{what}: top-1 differs on {mism.sum()} rows with margin >= 1e-4"
+    for k in ("max_prob", "margin") + (("cur_prob",) if "cur_prob" in got else ()):
+        err = np.abs(got[k] - ref[k][sel])
+        bound = P_ATOL + P_RTOL * np.abs(ref[k][sel])
+        assert (err <= bound).all(), f"{what}: {k} max err {err.max():.3e}"
+
+
+def test_scores_tiny_fp32(A):
+    z = synth.logits(64, 1024, seed=0, std=3.0, dtype="f32")
+    got = _run_scores(A, torch.from_numpy(z).cuda(), 1024)
+    assert_scores_close(got, O.decode_scores(z.astype(np.float64)), "tiny fp32")
+
+
+def test_scores_full_scoring_workload_bf16(A):
+    # [4 x 256 x 126464] bf16, N(0, 2.5^2) + planted U(0, 6): every row.
+    rows, V = 4 * 256, 126464
+    bits = synth.logits(rows, V, seed=0, std=2.5, boost_max=6.0)
+    mask = synth.mask_state(4, 256, seed=0).reshape(-1)
+    cur = synth.tokens(4, 256, V, seed=0, mask=mask.reshape(4, 256)).reshape(-1)
+    got = _run_scores(A, dev_bf16(bits), V, torch.from_numpy(mask).cuda(), torch.from_numpy(cur).cuda())
+    ref = O.decode_scores(synth.bf16_bits_to_f64(bits), mask_state=mask, cur_tokens=cur)
+    assert_scores_close(got, ref, "scoring workload")
+
+
+@pytest.mark.parametrize("V,stride,dtype", [(1001, 1008, "bf16"), (1001, 1004, "f32"), (1, 8, "bf16"),
+                                            (17, 20, "f32"), (40000, 40000, "bf16"), (33000, 33004, "f32"),
+                                            (152064, 152064, "bf16")])
+def test_scores_ragged_vocab_and_stride(A, V, stride, dtype):
+    rows = 24
+    z = synth.logits(rows, V, seed=5, std=2.0, boost_max=3.0, dtype=dtype)
+    zf = synth.bf16_bits_to_f64(z) if dtype == "bf16" else z.astype(np.float64)
+    zf[3, :] = 0.5                               # constant row: tie everywhere
+    zf[4, ::2] = -np.inf                         # half the vocabulary excluded
+    zf[5, :] = -np.inf
+    zf[5, V // 2] = 1.0                          # a single finite entry
+    pad = np.full((rows, stride), -np.inf)
+    pad[:, :V] = zf
+    if dtype == "bf16":
+        dev = dev_bf16(synth.to_bf16_bits(pad))
+    else:
+        dev = torch.from_numpy(pad.astype(np.float32)).cuda()
+    cur = np.arange(rows, dtype=np.int32) % V
+    got = _run_scores(A, dev, V, None, torch.from_numpy(cur).cuda())
+    ref = O.decode_scores(zf, cur_tokens=cur)
+    assert_scores_close(got, ref, f"V={V} {dtype}")
+    assert got["top1"][3] == 0 and got["top1"][5] == V // 2
+
+
+def test_scores_full_size_gqa_long_sampled(A):
+    rows, V = 16 * 512, 152064
+    z = synth.device_logits(rows, V, "cuda", seed=1, std=2.5)
+    got = _run_scores(A, z, V)
+    sample = np.unique(np.concatenate([[0, rows - 1], np.random.default_rng(1).integers(0, rows, 62)]))
+    ref = O.decode_scores(host_f64(z[torch.from_numpy(sample).cuda()]))
+    sub = {k: v[sample] for k, v in got.items()}
+    assert_scores_close(sub, ref, "gqa_long scoring (sampled rows)")
+
+
+def test_scores_workspace_reuse_is_clean(A):
+    # The ticket counters return to zero: repeated calls give identical results.
+    rows, V = 300, 70000
+    z = synth.device_logits(rows, V, "cuda", seed=2, std=2.0, boost_max=5.0)
+    first = _run_scores(A, z, V)
+    for _ in range(3):
+        again = _run_scores(A, z, V)
+        for k in first:
+            np.testing.assert_array_equal(first[k], again[k])
+
+
+# ----------------------------------------------------------------------------
+# refresh rule
+# ----------------------------------------------------------------------------
+
+@pytest.mark.parametrize("K,max_age", [(1, 0), (65, 8), (synth.K_INFINITE, 4), (0, 0), (3, 1)])
+def test_should_refresh_bit_exact(A, K, max_age):
+    rng = np.random.default_rng(K % 97 + max_age)
+    B, G = 37, 512
+    g = rng.integers(-1, 126464, size=(B, G)).astype(np.int32)
+    ga = g.copy()
+    for b in range(B):
+        n = rng.integers(0, 100)
+        pos = rng.choice(G, size=n, replace=False)
+        ga[b, pos] = ga[b, pos] + 1
+    age = rng.integers(0, 10, size=B).astype(np.int32)
+    for update in (False, True):
+        dg, dga, dage = (torch.from_numpy(a.copy()).cuda() for a in (g, ga, age))
+        dist = torch.empty(B, dtype=torch.int32, device="cuda")
+        flag = torch.empty(B, dtype=torch.uint8, device="cuda")
+        A.archer_should_refresh(dg, dga, dage, K, max_age, update, dist, flag)
+        torch.cuda.synchronize()
+        rd, rf, rga, rage = O.should_refresh(g, ga, age, K, max_age, update)
+        np.testing.assert_array_equal(dist.cpu().numpy(), rd)
+        np.testing.assert_array_equal(flag.cpu().numpy(), rf)
+        np.testing.assert_array_equal(dga.cpu().numpy(), rga)
+        np.testing.assert_array_equal(dage.cpu().numpy(), rage)
