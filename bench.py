@@ -1,0 +1,497 @@
+"""Benchmark of the Archer denoising step on one GB300 (or N replicas).
+
+A "step" is one pass of the whole hot path over one batch: the redraw that
+stands in for the rollback decoder, the refresh rule (archer_should_refresh),
+the refresh-flag read-back, attention in every layer (archer_attn_step, or
+archer_prompt_refresh with the prompt-cache rewrite when the rule fires) and
+decoder scoring (archer_decode_scores).  Default workload: the long-prompt GQA
+trajectory (batch 16, 28 query / 4 KV heads, head_dim 128, prompt 4096,
+response 512, 32 layers, 5% redraw per step, refresh every 16 steps, scoring
+over a 152064-token vocabulary).
+
+Reported on one JSON line (rank 0):
+  value        denoise steps/s over K timed steps (device inputs resident in HBM)
+  e2e          the same through the C ABI with every step's inputs copied from
+               pinned host memory and the scores copied back
+  roofline     the attention kernel: algorithmic FLOPs per launch / mean launch
+               time (CUDA events on the launching stream) vs the measured bf16 peak
+  speedup_vs_refresh_every_step   against the eager arm (refresh at every step)
+  scoring      decode_scores GB/s vs the measured HBM copy bandwidth
+  cpu_baseline the fp64 oracle on a bounded sample, on this host's cores
+Every input is larger than L2 (each layer's prompt K/V alone exceeds 129 MB),
+so no explicit L2 flush is done between steps.
+
+--impl reference times the oracle (the CPU reference of this build) on bounded
+samples of the same workload.  Multi-GPU (torchrun): independent replicas, one
+per rank, no collective on the data path ("scaling": "weak").
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+import torch  # noqa: E402
+
+from paper_2608_08086_gb300 import synth  # noqa: E402
+
+METRIC = "denoise steps/s"
+PEAKS_FALLBACK = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+
+
+def peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            p = json.load(f)
+        return p, "measured"
+    except (OSError, ValueError):
+        return PEAKS_FALLBACK, "fallback"
+
+
+# ---------------------------------------------------------------------------- clocks
+
+class ClockSampler:
+    """nvidia-smi clocks and throttle reasons, sampled every 200 ms."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.path = None
+
+    def start(self):
+        fd, self.path = tempfile.mkstemp(suffix=".csv")
+        os.close(fd)
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-lms", "200"], stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+        except OSError:
+            self.proc = None
+
+    def stop(self):
+        out = {"sm_mhz": None, "sm_max_mhz": None, "reasons": [], "samples": 0}
+        if self.proc is None:
+            return out
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        rows = []
+        with open(self.path) as f:
+            for line in f:
+                parts = [p.strip() for p in line.split(",")]
+                if len(parts) >= 9:
+                    rows.append(parts)
+        os.unlink(self.path)
+        if not rows:
+            return out
+        sm = [float(r[1]) for r in rows if r[1].replace(".", "").isdigit()]
+        out["samples"] = len(rows)
+        out["sm_mhz"] = statistics.median(sm) if sm else None
+        out["sm_max_mhz"] = max(float(r[2]) for r in rows if r[2].replace(".", "").isdigit()) if sm else None
+        names = ("hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap")
+        reasons = set()
+        for r in rows:
+            for name, v in zip(names, r[5:9]):
+                if v.lower() == "active":
+                    reasons.add(name)
+        out["reasons"] = sorted(reasons)
+        return out
+
+
+# ---------------------------------------------------------------------------- timing helpers
+
+def barrier(dist_on):
+    if dist_on:
+        torch.distributed.barrier()
+    torch.cuda.synchronize()
+
+
+def max_over_ranks(x: float, dist_on: bool) -> float:
+    if not dist_on:
+        return x
+    t = torch.tensor([x], dtype=torch.float64, device="cuda")
+    torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
+    return float(t.item())
+
+
+def run_arm(wl, mode, steps, warmup, dist_on, time_attention=False, seed=0):
+    from paper_2608_08086_gb300.trajectory import DeviceTrajectory
+    tr = DeviceTrajectory(wl, seed=seed, mode=mode, source="device", max_steps=warmup + steps + 1)
+    tr.build()
+    for _ in range(warmup):
+        tr.step()
+    barrier(dist_on)
+    tr.time_attention = time_attention
+    tr.attn_events = []
+    refresh_before = tr.n_refresh_steps
+    start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    torch.cuda.nvtx.range_push(f"timed-{mode}")
+    start.record()
+    for _ in range(steps):
+        tr.step()
+    end.record()
+    torch.cuda.nvtx.range_pop()
+    barrier(dist_on)
+    ms = start.elapsed_time(end)
+    info = {"ms": ms, "refresh_steps": tr.n_refresh_steps - refresh_before, "traj": tr}
+    return info
+
+
+def kernel_only(args, wl):
+    """A few launches of one kernel on the workload's full-size tensors (for
+    profiler captures): attn_step | attn_refresh | scores."""
+    from paper_2608_08086_gb300 import archer as A
+    sh = wl.shape
+    B, P, G, Hq, Hkv, D = sh.batch, sh.prompt_len, sh.resp_len, sh.n_heads, sh.n_kv_heads, sh.head_dim
+    dev = torch.device("cuda")
+    if args.kernel_only.startswith("attn"):
+        d = synth.device_attn_inputs(sh, dev, seed=0)
+        shape = A.make_shape(B, P, G, Hq, Hkv, D)
+        if args.kernel_only == "attn_step":
+            q = d["q_all"][:, P:].contiguous()
+            out = torch.empty(B, G, Hq, D, dtype=torch.bfloat16, device=dev)
+            fn = lambda: A.archer_attn_step(shape, q, d["k_cache"], d["v_cache"], d["k_resp"], d["v_resp"], out)  # noqa: E731
+        else:
+            out = torch.empty(B, P + G, Hq, D, dtype=torch.bfloat16, device=dev)
+            fn = lambda: A.archer_prompt_refresh(shape, d["q_all"], d["k_prompt"], d["v_prompt"], d["k_resp"],  # noqa: E731
+                                                 d["v_resp"], out, None, d["k_prompt"], d["v_prompt"])
+    else:
+        rows = wl.logits_rows
+        z = synth.device_logits(rows, wl.vocab, dev, seed=0, std=wl.logits_std, boost_max=wl.logits_boost)
+        mp = torch.empty(rows, dtype=torch.float32, device=dev)
+        t1 = torch.empty(rows, dtype=torch.int32, device=dev)
+        mg = torch.empty(rows, dtype=torch.float32, device=dev)
+        fn = lambda: A.archer_decode_scores(z, mp, t1, mg)  # noqa: E731
+    for _ in range(args.warmup):
+        fn()
+    torch.cuda.synchronize()
+    start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    start.record()
+    for _ in range(args.launches):
+        fn()
+    end.record()
+    torch.cuda.synchronize()
+    A.archer_check_device()
+    print(json.dumps({"kernel_only": args.kernel_only, "workload": wl.name, "launches": args.launches,
+                      "mean_ms": start.elapsed_time(end) / args.launches}), flush=True)
+    return 0
+
+
+def kernel_stats(tr):
+    """Mean durations (ms) and counts of the attention / scoring launches."""
+    by = {}
+    for s, e, kind in tr.attn_events:
+        by.setdefault(kind, []).append(s.elapsed_time(e))
+    return {k: {"count": len(v), "mean_ms": sum(v) / len(v), "total_ms": sum(v)} for k, v in by.items()}
+
+
+# ---------------------------------------------------------------------------- e2e
+
+def run_e2e(wl, steps, warmup, dist_on, seed=0):
+    """The same step through the C ABI with HOST inputs: every step copies its
+    inputs (token updates, redrawn Q/K/V rows of every layer, the step's logits,
+    and at a refresh the fresh prompt Q/K/V of every layer) from pinned host
+    memory, and reads the scores back."""
+    from paper_2608_08086_gb300.trajectory import DeviceTrajectory
+    tr = DeviceTrajectory(wl, seed=seed, mode="archer", source="device", max_steps=warmup + steps + 1)
+    sh = wl.shape
+    B, P, G, Hq, Hkv, D, L = sh.batch, sh.prompt_len, sh.resp_len, sh.n_heads, sh.n_kv_heads, sh.head_dim, tr.L
+    n = wl.redraws_per_step
+    # host staging buffers (pinned): one layer's worth, copied to every layer
+    h_rows_q = tr.pool["q"][0].cpu().pin_memory()          # [L, B, n, Hq, D]
+    h_rows_k = tr.pool["k"][0].cpu().pin_memory()
+    h_rows_v = tr.pool["v"][0].cpu().pin_memory()
+    h_logits = tr.logits.cpu().pin_memory()
+    h_q_prompt = tr.q_all[0][:, :P].contiguous().cpu().pin_memory()
+    h_k_new = tr.k_new[0].cpu().pin_memory()
+    h_v_new = tr.v_new[0].cpu().pin_memory()
+    h_scores = torch.empty(3, B * G, dtype=torch.float32).pin_memory()
+    d_rows = {c: torch.empty_like(tr.pool[c][0]) for c in ("q", "k", "v")}
+    plan_host = [(p.cpu().pin_memory(), v.cpu().pin_memory()) for p, v in tr.plan]
+    d_pos = torch.empty_like(tr.plan[0][0])
+    d_new = torch.empty_like(tr.plan[0][1])
+    bytes_in = {"step": 0, "refresh": 0}
+
+    orig_stage = tr._stage_redraw
+    orig_fresh = tr._stage_fresh_prompt
+
+    def stage_redraw(t):
+        hp, hn = plan_host[(t - 1) % len(plan_host)]
+        d_pos.copy_(hp, non_blocking=True)
+        d_new.copy_(hn, non_blocking=True)
+        for c, h in (("q", h_rows_q), ("k", h_rows_k), ("v", h_rows_v)):
+            d_rows[c].copy_(h, non_blocking=True)
+        tr.logits.copy_(h_logits, non_blocking=True)
+        bidx = torch.arange(B, device=tr.device)[:, None]
+        tr.g[bidx, d_pos] = d_new
+        tr.q_resp[:, bidx, d_pos] = d_rows["q"]
+        tr.q_all[:, bidx, P + d_pos] = d_rows["q"]
+        tr.k_resp[:, bidx, d_pos] = d_rows["k"]
+        tr.v_resp[:, bidx, d_pos] = d_rows["v"]
+
+    def stage_fresh(t):
+        for layer in range(L):
+            tr.q_all[layer][:, :P].copy_(h_q_prompt, non_blocking=True)
+            tr.k_new[layer].copy_(h_k_new, non_blocking=True)
+            tr.v_new[layer].copy_(h_v_new, non_blocking=True)
+
+    tr._stage_redraw = stage_redraw
+    tr._stage_fresh_prompt = stage_fresh
+    nb = lambda t: t.numel() * t.element_size()  # noqa: E731
+    per_step_in = (nb(plan_host[0][0]) + nb(plan_host[0][1]) + nb(h_rows_q) + nb(h_rows_k) + nb(h_rows_v)
+                   + nb(h_logits))
+    per_refresh_in = L * (nb(h_q_prompt) + nb(h_k_new) + nb(h_v_new))
+    tr.build()
+    for _ in range(warmup):
+        tr.step()
+        h_scores[0].copy_(tr.max_prob, non_blocking=True)
+    barrier(dist_on)
+    r0 = tr.n_refresh_steps
+    start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    start.record()
+    for _ in range(steps):
+        tr.step()
+        h_scores[0].copy_(tr.max_prob, non_blocking=True)
+        h_scores[1].copy_(tr.top1.view(torch.float32), non_blocking=True)
+        h_scores[2].copy_(tr.margin, non_blocking=True)
+    end.record()
+    barrier(dist_on)
+    ms = start.elapsed_time(end)
+    n_ref = tr.n_refresh_steps - r0
+    h2d = (steps * per_step_in + n_ref * per_refresh_in) / steps
+    d2h = B + 3 * B * G * 4      # the refresh flags and the three score vectors
+    del tr
+    torch.cuda.empty_cache()
+    return {"ms": ms, "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h)}
+
+
+# ---------------------------------------------------------------------------- oracle (CPU)
+
+def oracle_sample_step(wl, n_pairs=None, score_rows=8, seed=0):
+    """One bounded sample of a step on the fp64 oracle, extrapolated to the full
+    step: cached attention of `n_pairs` (sequence, head) pairs of one layer, one
+    refresh pair, and scoring of `score_rows` rows; scaled by the workload's
+    pair, layer and row counts and its refresh fraction.  Returns
+    (seconds per full step, sample description, threads)."""
+    from oracle import oracle as O
+    sh = wl.shape
+    B, P, G, Hq, Hkv, D = sh.batch, sh.prompt_len, sh.resp_len, sh.n_heads, sh.n_kv_heads, sh.head_dim
+    threads = O.hardware_threads()
+    n_pairs = n_pairs or max(1, threads)
+    rng = np.random.default_rng(seed)
+    std = 1.0 / math.sqrt(D)
+    q = rng.standard_normal((1, G, n_pairs, D)) * std
+    kc = rng.standard_normal((1, P, n_pairs, D)) * std
+    vc = rng.standard_normal((1, P, n_pairs, D)) * std
+    kg = rng.standard_normal((1, G, n_pairs, D)) * std
+    vg = rng.standard_normal((1, G, n_pairs, D)) * std
+    t0 = time.perf_counter()
+    O.attention(q, kc, vc, kg, vg, 1.0 / math.sqrt(D), n_threads=threads)      # n_pairs independent heads
+    t_cached_pairs = time.perf_counter() - t0
+    # refresh costs N/G times a cached pair (N queries instead of G)
+    t_refresh_pair = t_cached_pairs / n_pairs * (P + G) / G
+    t_score = 0.0
+    if wl.logits_rows:
+        z = rng.standard_normal((score_rows, wl.vocab)) * wl.logits_std
+        t0 = time.perf_counter()
+        O.decode_scores(z, n_threads=threads)
+        t_score = (time.perf_counter() - t0) / score_rows * wl.logits_rows
+    pairs = B * Hq
+    q_k = 1.0 / wl.max_age if wl.max_age else 1.0 / 3.0
+    per_layer = (1 - q_k) * t_cached_pairs / n_pairs * pairs + q_k * t_refresh_pair * pairs
+    step_s = wl.layers * per_layer + t_score
+    sample = (f"{n_pairs} (sequence, head) pairs of one cached layer ({G} queries x {P + G} keys, D={D}) and "
+              f"{score_rows} scoring rows of {wl.vocab}, extrapolated to {pairs} pairs x {wl.layers} layers with "
+              f"refresh fraction {q_k:.3f} and {wl.logits_rows} rows")
+    return step_s, sample, threads
+
+
+def reference_arm(args, wl):
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return 0
+    for _ in range(args.warmup):
+        oracle_sample_step(wl, n_pairs=4, score_rows=2)
+    times = []
+    sample = ""
+    threads = 0
+    for _ in range(args.steps):
+        s, sample, threads = oracle_sample_step(wl, n_pairs=4, score_rows=2)
+        times.append(s)
+    step_s = statistics.median(times)
+    value = 1.0 / step_s
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": "steps/s", "n_gpus": args.gpus,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": step_s * 1e3, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": {"workload": wl.name},
+            "cpu_baseline": {"kind": "oracle", "value": value, "unit": "steps/s", "cores": threads,
+                             "sample": sample + " per step (extrapolated)"},
+            "e2e": {"value": value, "unit": "steps/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+# ---------------------------------------------------------------------------- main
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--workload", default="gqa_long", choices=["gqa_long", "traj32"])
+    ap.add_argument("--eager-steps", type=int, default=4)
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu", action="store_true")
+    ap.add_argument("--no-secondary", action="store_true")
+    ap.add_argument("--kernel-only", choices=["attn_step", "attn_refresh", "scores"], default=None,
+                    help="run only a few launches of one kernel (for profiler captures)")
+    ap.add_argument("--launches", type=int, default=3)
+    args = ap.parse_args()
+    args.warmup = max(args.warmup, 3)
+    wl = synth.WORKLOADS[args.workload]
+
+    if args.impl == "reference":
+        return reference_arm(args, wl)
+    if args.kernel_only:
+        torch.cuda.set_device(int(os.environ.get("LOCAL_RANK", "0")))
+        from paper_2608_08086_gb300 import build as Bld
+        Bld.build()
+        return kernel_only(args, wl)
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    dist_on = world > 1
+    torch.cuda.set_device(local)
+    if dist_on:
+        torch.distributed.init_process_group("nccl", device_id=torch.device("cuda", local))
+
+    from paper_2608_08086_gb300 import build as B
+    B.build()
+    from paper_2608_08086_gb300 import archer as A  # noqa: F401  (fails loudly without libarcher)
+
+    pk, pk_kind = peaks()
+    clocks = ClockSampler(local)
+
+    # ---- the Archer arm (timed region = K steps)
+    clocks.start()
+    arm = run_arm(wl, "archer", args.steps, args.warmup, dist_on, time_attention=True)
+    clk = clocks.stop()
+    tr = arm["traj"]
+    ms = max_over_ranks(arm["ms"], dist_on)
+    value = world * args.steps / (ms / 1e3)
+    ks = kernel_stats(tr)
+    L = tr.L
+    n_ref = arm["refresh_steps"]
+    launches = args.steps * (1 + L + (1 if tr.score else 0)) + n_ref * L   # rule + attention + scoring + rewrites
+    flops_step_launch = 4.0 * tr.B * tr.Hq * tr.G * tr.N * tr.D
+    flops_refresh_launch = 4.0 * tr.B * tr.Hq * tr.N * tr.N * tr.D
+    att = {}
+    tot_flops, tot_ms = 0.0, 0.0
+    for kind, fl in (("step", flops_step_launch), ("refresh", flops_refresh_launch)):
+        if kind in ks:
+            k = ks[kind]
+            att[kind] = {"launches": k["count"], "mean_ms": k["mean_ms"], "tflops": fl / (k["mean_ms"] * 1e9)}
+            tot_flops += fl * k["count"]
+            tot_ms += k["total_ms"]
+    peak_tf = pk["bf16_tflops_sustained"]
+    achieved = tot_flops / (tot_ms * 1e9) if tot_ms else 0.0
+    scoring = None
+    if "score" in ks:
+        sbytes = tr.B * tr.G * wl.vocab * (2 if wl.logits_dtype == "bf16" else 4)
+        gbs = sbytes / (ks["score"]["mean_ms"] * 1e6)
+        scoring = {"mean_ms": ks["score"]["mean_ms"], "gbs": gbs, "peak_gbs": pk["hbm_gbs"],
+                   "frac": gbs / pk["hbm_gbs"], "bytes_per_launch": sbytes}
+    del arm, tr
+    torch.cuda.empty_cache()
+
+    # ---- the eager arm: refresh every step
+    eager = run_arm(wl, "eager", args.eager_steps, 3, dist_on)
+    eager_ms = max_over_ranks(eager["ms"], dist_on)
+    eager_value = world * args.eager_steps / (eager_ms / 1e3)
+    del eager
+    torch.cuda.empty_cache()
+
+    # ---- e2e through host buffers
+    e2e = None
+    if not args.no_e2e:
+        e = run_e2e(wl, args.steps, args.warmup, dist_on)
+        e_ms = max_over_ranks(e["ms"], dist_on)
+        e2e = {"value": world * args.steps / (e_ms / 1e3), "unit": "steps/s",
+               "h2d_bytes_per_step": e["h2d_bytes_per_step"], "d2h_bytes_per_step": e["d2h_bytes_per_step"]}
+
+    # ---- a second trajectory workload (32 layers, B 8, P 1024, G 512, rule K=65 / age 8)
+    secondary = None
+    if not args.no_secondary and args.workload != "traj32":
+        wl2 = synth.WORKLOADS["traj32"]
+        a2 = run_arm(wl2, "archer", min(args.steps, 30), 3, dist_on, time_attention=True)
+        ks2 = kernel_stats(a2["traj"])
+        e2 = run_arm(wl2, "eager", args.eager_steps, 3, dist_on)
+        v2 = world * min(args.steps, 30) / (max_over_ranks(a2["ms"], dist_on) / 1e3)
+        ve2 = world * args.eager_steps / (max_over_ranks(e2["ms"], dist_on) / 1e3)
+        t2 = a2["traj"]
+        fl2 = 4.0 * t2.B * t2.Hq * t2.G * t2.N * t2.D
+        secondary = {"workload": wl2.name, "steps_per_s": v2, "eager_steps_per_s": ve2, "speedup_vs_refresh_every_step": v2 / ve2,
+                     "refresh_steps": a2["refresh_steps"],
+                     "step_attention_tflops": fl2 / (ks2["step"]["mean_ms"] * 1e9) if "step" in ks2 else None}
+        del a2, e2, t2
+        torch.cuda.empty_cache()
+
+    # ---- CPU baseline: the oracle on a bounded sample (rank 0, N = 1)
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu:
+        s, sample, threads = oracle_sample_step(wl)
+        cpu = {"value": 1.0 / s, "unit": "steps/s", "cores": threads, "kind": "oracle", "sample": sample}
+
+    if rank == 0:
+        line = {
+            "metric": METRIC, "value": value, "unit": "steps/s", "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": ms / args.steps, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+            "config": {"workload": wl.name, "batch": wl.shape.batch, "prompt_len": wl.shape.prompt_len,
+                       "resp_len": wl.shape.resp_len, "n_heads": wl.shape.n_heads, "n_kv_heads": wl.shape.n_kv_heads,
+                       "head_dim": wl.shape.head_dim, "layers": wl.layers, "vocab": wl.vocab,
+                       "redraws_per_step": wl.redraws_per_step, "max_age": wl.max_age,
+                       "radius_k": None if wl.radius_k >= synth.K_INFINITE else wl.radius_k,
+                       "parallelism": f"replicas{world}" if world > 1 else "single",
+                       "l2": "no flush: inputs larger than L2 (prompt K/V of one layer > 129 MB)"},
+            "refresh_steps_timed": n_ref,
+            "speedup_vs_refresh_every_step": value / eager_value,
+            "eager_steps_per_s": eager_value,
+            "attention": att,
+            "roofline": {"bound": "tensor", "kernel": "attn_fwd_kernel<128>", "achieved": achieved, "peak": peak_tf,
+                         "unit": "TFLOP/s", "frac": achieved / peak_tf, "traffic": None,
+                         "peak_kind": f"bf16_tflops_sustained ({pk_kind})"},
+            "scoring": scoring,
+            "e2e": e2e,
+            "gpu_launches": launches,
+            "clocks": {"sm_mhz": clk["sm_mhz"], "sm_max_mhz": clk["sm_max_mhz"], "reasons": clk["reasons"]},
+            "secondary": secondary,
+            "cpu_baseline": cpu,
+        }
+        print(json.dumps(line), flush=True)
+    if dist_on:
+        torch.distributed.destroy_process_group()
+    return 0
+
+
+if __name__ == "__main__":
+    sys.exit(main())

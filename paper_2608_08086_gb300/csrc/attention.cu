@@ -59,8 +59,8 @@ struct Layout {
   static constexpr uint32_t kOffK = kOffQ + kTile;
   static constexpr uint32_t kOffV = kOffK + kKS * kTile;
   static constexpr uint32_t kOffBar = kOffV + kVS * kTile;
-  // q_full, k_full[KS], k_empty[KS], v_full[VS], v_empty[VS], s_full[2], p_full[2], pv_done
-  static constexpr int kBars = 1 + 2 * kKS + 2 * kVS + 2 + 2 + 1;
+  // q_full, k_full[KS], k_empty[KS], v_full[VS], v_empty[VS], s_full[2], p_full[2], pv_done[2]
+  static constexpr int kBars = 1 + 2 * kKS + 2 * kVS + 2 + 2 + 2;
   static constexpr uint32_t kOffHolder = kOffBar + 8 * kBars;
   static constexpr uint32_t kOffAbort = kOffHolder + 4;
   static constexpr uint32_t kUsed = kOffAbort + 4;
@@ -122,7 +122,7 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
   const uint32_t bar_v_empty = bar_v_full + 8 * L::kVS;
   const uint32_t bar_s_full = bar_v_empty + 8 * L::kVS;         // + 8 * buffer
   const uint32_t bar_p_full = bar_s_full + 16;
-  const uint32_t bar_pv_done = bar_p_full + 16;
+  const uint32_t bar_pv_done = bar_p_full + 16;                 // + 8 * (tile & 1)
   uint32_t* holder = reinterpret_cast<uint32_t*>(gbase + L::kOffHolder);
   volatile int* abort = reinterpret_cast<volatile int*>(gbase + L::kOffAbort);
 
@@ -140,8 +140,8 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
     for (int i = 0; i < 2; ++i) {
       mbar_init(bar_s_full + 8 * i, 1);
       mbar_init(bar_p_full + 8 * i, kBM);
+      mbar_init(bar_pv_done + 8 * i, 1);
     }
-    mbar_init(bar_pv_done, 1);
     *abort = 0;
     mbar_fence_init();
   }
@@ -225,7 +225,7 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
         if (!mbar_wait(bar_p_full + 8 * (j & 1), (j >> 1) & 1, abort, p.err)) break;
         tc_fence_after();
         issue_pv((j & 1) ? kColP1 : kColP0, sV + vs * L::kTile, j > 0);
-        umma_commit(bar_pv_done);
+        umma_commit(bar_pv_done + 8 * (j & 1));
         umma_commit(bar_v_empty + 8 * vs);
       }
     }
@@ -261,16 +261,23 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
       const float tmax = fmaxf(fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3])),
                                fmaxf(fmaxf(mx[4], mx[5]), fmaxf(mx[6], mx[7])));
       const float mt2 = tmax * sl2;
-      if (j > 0) {
-        // PV_{j-1} done: O is stable and P[sb] (last read by PV_{j-2}) is free.
-        if (!warp_wait(bar_pv_done, (j - 1) & 1, abort, p.err)) { ok = false; break; }
+      // PV_j commits to pv_done[j & 1], so each barrier's next phase belongs to
+      // a PV that needs this thread's next P: no wait below can see its
+      // barrier two phases ahead.
+      if (j >= 2) {
+        // P[sb] was last read by PV_{j-2}.
+        if (!warp_wait(bar_pv_done + 8 * sb, ((j - 2) >> 1) & 1, abort, p.err)) { ok = false; break; }
         tc_fence_after();
       }
       if (j == 0) {
         m_used = mt2;
-      } else if (mt2 > m_used + 8.0f) {
-        const float alpha = ex2_approx(m_used - mt2);
-        m_used = mt2;
+      } else if (__any_sync(0xffffffffu, mt2 > m_used + 8.0f)) {
+        // Rescale O: wait until PV_{j-1} has finished accumulating into it.
+        if (!warp_wait(bar_pv_done + 8 * (sb ^ 1), ((j - 1) >> 1) & 1, abort, p.err)) { ok = false; break; }
+        tc_fence_after();
+        const float m_new = fmaxf(m_used, mt2);
+        const float alpha = ex2_approx(m_used - m_new);
+        m_used = m_new;
         l_sum *= alpha;
 #pragma unroll
         for (int c0 = 0; c0 < D; c0 += 32) {
@@ -296,7 +303,7 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
       tc_fence_before();
       mbar_arrive(bar_p_full + 8 * sb);
     }
-    if (ok && warp_wait(bar_pv_done, (T - 1) & 1, abort, p.err)) {
+    if (ok && warp_wait(bar_pv_done + 8 * ((T - 1) & 1), ((T - 1) >> 1) & 1, abort, p.err)) {
       tc_fence_after();
       const float inv_l = 1.0f / l_sum;
       const int q = q0 + r;

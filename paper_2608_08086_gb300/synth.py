@@ -327,3 +327,61 @@ def device_logits(rows: int, vocab: int, device, seed: int = 0, std: float = 2.5
                      dtype=torch.bfloat16 if dtype is None else dtype)
     out[:, :vocab] = z.to(out.dtype)
     return out
+
+
+# ----------------------------------------------------------------------------
+# trajectory inputs (Algorithm 1 with the rollback decoder replaced by a
+# seeded redraw).  Step 0 builds the cache; at step t >= 1, n positions per
+# sequence get a new token id and new Q/K/V rows in every layer.  Fresh prompt
+# Q/K/V (the stand-in for the model's prompt states under the current
+# response) are drawn per (layer, step) and used only when a refresh fires.
+# ----------------------------------------------------------------------------
+
+def traj_initial_tokens(wl: Workload, seed: int = 0) -> np.ndarray:
+    sh = wl.shape
+    m = mask_state(sh.batch, sh.resp_len, seed=seed)
+    return tokens(sh.batch, sh.resp_len, max(wl.vocab, 2), seed=seed, mask=m)
+
+
+def traj_layer_initial(wl: Workload, seed: int, layer: int) -> dict:
+    """Step-0 bits of one layer: q_all [B,N,Hq,D], k_resp/v_resp [B,G,Hkv,D],
+    k_new/v_new [B,P,Hkv,D] (the fresh prompt K/V of the build)."""
+    x = attn_inputs(wl.shape, seed=seed, layer=layer, step=0)
+    return {"q_all": x["q_all"], "k_resp": x["k_resp"], "v_resp": x["v_resp"],
+            "k_new": x["k_prompt"], "v_new": x["v_prompt"]}
+
+
+def traj_redraw(wl: Workload, seed: int, step: int, g_current: np.ndarray):
+    """Positions [B, n] (sorted, distinct) and their new token ids [B, n]."""
+    B, G = g_current.shape
+    n = wl.redraws_per_step
+    pos = np.stack([redraw_positions(seed, step, b, G, n) for b in range(B)]) if n else np.zeros((B, 0), np.int64)
+    new = np.stack([redraw_tokens(seed, step, b, g_current[b, pos[b]], max(wl.vocab, 2)) for b in range(B)]) \
+        if n else np.zeros((B, 0), np.int32)
+    return pos, new
+
+
+def traj_redraw_rows(wl: Workload, seed: int, step: int, layer: int) -> dict:
+    """New bf16 rows for the redrawn positions: q [B,n,Hq,D], k/v [B,n,Hkv,D]."""
+    sh = wl.shape
+    n = wl.redraws_per_step
+    std = 1.0 / math.sqrt(sh.head_dim)
+    return {"q": redraw_rows(seed, step, layer, "q", (sh.batch, n, sh.n_heads, sh.head_dim), std),
+            "k": redraw_rows(seed, step, layer, "k", (sh.batch, n, sh.n_kv_heads, sh.head_dim), std),
+            "v": redraw_rows(seed, step, layer, "v", (sh.batch, n, sh.n_kv_heads, sh.head_dim), std)}
+
+
+def traj_fresh_prompt(wl: Workload, seed: int, step: int, layer: int) -> dict:
+    """Fresh prompt queries [B,P,Hq,D] and K/V [B,P,Hkv,D] at a refresh of step t."""
+    sh = wl.shape
+    std = 1.0 / math.sqrt(sh.head_dim)
+    tag = ("fresh-prompt", seed, step, layer)
+    return {"q_prompt": bf16_normal(tag + ("q",), (sh.batch, sh.prompt_len, sh.n_heads, sh.head_dim), std),
+            "k_new": bf16_normal(tag + ("k",), (sh.batch, sh.prompt_len, sh.n_kv_heads, sh.head_dim), std),
+            "v_new": bf16_normal(tag + ("v",), (sh.batch, sh.prompt_len, sh.n_kv_heads, sh.head_dim), std)}
+
+
+def traj_logits(wl: Workload, seed: int, step: int):
+    """Logits scored after the forward of step t: [B*G, V] bf16 bits or fp32."""
+    return logits(wl.shape.batch * wl.shape.resp_len, wl.vocab, seed=seed, std=wl.logits_std,
+                  boost_max=wl.logits_boost, dtype=wl.logits_dtype, step=step)

@@ -1,0 +1,237 @@
+"""Algorithm 1 (state-anchored rollback decoding) driven through the C ABI.
+
+The rollback decoder D is replaced by the seeded redraw of ``synth`` (a fixed
+number of response positions per sequence get a new token and new Q/K/V rows
+in every layer each step).  Per step t:
+
+  1. stage the redraw (token ids and Q/K/V rows)           -- stands in for D
+  2. archer_should_refresh: D_t = d_H(g_t, g_r), flag = D_t >= K or age_t >= max_age;
+     flagged sequences take g_r <- g_t, age <- 0 (Sec. 4.2, Eq. archer-controller)
+  3. the flags are read back to the host (one 1-byte-per-sequence copy)
+  4. per layer: archer_prompt_refresh (if any flag; per-sequence flags, prompt
+     cache rewritten) or archer_attn_step (Eq. archer-cached)
+  5. archer_decode_scores over the step's logits.
+Step 0 is the FullForward that builds every layer's prompt cache.
+``mode="eager"`` refreshes every step (K = 0), the full-recomputation comparator.
+
+Per-layer buffers are slices of stacked tensors so that one indexed copy
+stages a redraw for all layers.  With ``source="host"`` every input comes
+from the host generator of ``synth`` (bit-identical to what the oracle sees);
+with ``source="device"`` inputs are drawn on the GPU once, and redraw rows come
+from a pre-drawn pool (cycled), so that all inputs are resident in HBM.
+"""
+from __future__ import annotations
+
+import math
+
+import numpy as np
+import torch
+
+from . import archer as A
+from . import synth
+
+
+def _dev_bits(bits, device):
+    return torch.from_numpy(np.ascontiguousarray(bits).view(np.int16)).view(torch.bfloat16).to(device)
+
+
+class DeviceTrajectory:
+    def __init__(self, wl: synth.Workload, seed: int = 0, mode: str = "archer", source: str = "host",
+                 device="cuda", layers: int | None = None, score: bool = True, pool_steps: int = 8,
+                 max_steps: int | None = None, record: bool = False):
+        self.wl, self.seed, self.mode, self.source = wl, seed, mode, source
+        self.device = torch.device(device)
+        sh = wl.shape
+        self.B, self.P, self.G = sh.batch, sh.prompt_len, sh.resp_len
+        self.Hq, self.Hkv, self.D = sh.n_heads, sh.n_kv_heads, sh.head_dim
+        self.N = self.P + self.G
+        self.L = wl.layers if layers is None else layers
+        self.K = 0 if mode == "eager" else wl.radius_k
+        self.max_age = 0 if mode == "eager" else wl.max_age
+        self.score = score and wl.logits_rows > 0
+        self.record = record
+        self.shape = A.make_shape(self.B, self.P, self.G, self.Hq, self.Hkv, self.D)
+        self.pool_steps = pool_steps
+        self.max_steps = wl.steps if max_steps is None else max_steps
+        self.n_refresh_steps = 0
+        self.t = -1
+        self.attn_events = []          # (start, end, kind) CUDA events around attention launches
+        self.time_attention = False
+        self._alloc()
+
+    # ------------------------------------------------------------------ setup
+    def _alloc(self):
+        B, P, G, N, Hq, Hkv, D, L = self.B, self.P, self.G, self.N, self.Hq, self.Hkv, self.D, self.L
+        dev, bf = self.device, torch.bfloat16
+        std = 1.0 / math.sqrt(D)
+        if self.source == "host":
+            g0 = synth.traj_initial_tokens(self.wl, self.seed)
+            init = [synth.traj_layer_initial(self.wl, self.seed, layer) for layer in range(L)]
+            self.q_all = torch.stack([_dev_bits(x["q_all"], dev) for x in init])
+            self.k_resp = torch.stack([_dev_bits(x["k_resp"], dev) for x in init])
+            self.v_resp = torch.stack([_dev_bits(x["v_resp"], dev) for x in init])
+            self.k_new = torch.stack([_dev_bits(x["k_new"], dev) for x in init])
+            self.v_new = torch.stack([_dev_bits(x["v_new"], dev) for x in init])
+            self.g_host = g0.copy()
+        else:
+            tag = ("traj-dev", self.seed)
+            self.q_all = synth.device_normal(tag + ("q",), (L, B, N, Hq, D), std, dev)
+            self.k_resp = synth.device_normal(tag + ("kg",), (L, B, G, Hkv, D), std, dev)
+            self.v_resp = synth.device_normal(tag + ("vg",), (L, B, G, Hkv, D), std, dev)
+            self.k_new = synth.device_normal(tag + ("kp",), (L, B, P, Hkv, D), std, dev)
+            self.v_new = synth.device_normal(tag + ("vp",), (L, B, P, Hkv, D), std, dev)
+            self.g_host = synth.traj_initial_tokens(self.wl, self.seed)
+            n = self.wl.redraws_per_step
+            self.pool = {
+                "q": synth.device_normal(tag + ("pool-q",), (self.pool_steps, L, B, n, Hq, D), std, dev),
+                "k": synth.device_normal(tag + ("pool-k",), (self.pool_steps, L, B, n, Hkv, D), std, dev),
+                "v": synth.device_normal(tag + ("pool-v",), (self.pool_steps, L, B, n, Hkv, D), std, dev),
+            }
+            # the token trajectory is cheap: plan it on the host for every step
+            self.plan = []
+            g = self.g_host.copy()
+            for t in range(1, self.max_steps + 1):
+                pos, new = synth.traj_redraw(self.wl, self.seed, t, g)
+                g[np.arange(B)[:, None], pos] = new
+                self.plan.append((torch.from_numpy(pos).to(dev), torch.from_numpy(new).to(dev)))
+        self.q_resp = self.q_all[:, :, P:].contiguous()
+        self.k_cache = torch.zeros_like(self.k_new)
+        self.v_cache = torch.zeros_like(self.v_new)
+        self.g = torch.from_numpy(self.g_host).to(dev)
+        self.g_anchor = self.g.clone()
+        self.age = torch.zeros(B, dtype=torch.int32, device=dev)
+        self.dist = torch.zeros(B, dtype=torch.int32, device=dev)
+        self.flag = torch.ones(B, dtype=torch.uint8, device=dev)
+        self.flag_host = torch.ones(B, dtype=torch.uint8).pin_memory()
+        self.out_step = torch.empty(B, G, Hq, D, dtype=bf, device=dev)
+        self.out_full = torch.empty(B, N, Hq, D, dtype=bf, device=dev)
+        if self.score:
+            rows, V = B * G, self.wl.vocab
+            if self.source == "host":
+                self.logits = None
+            else:
+                dt = torch.bfloat16 if self.wl.logits_dtype == "bf16" else torch.float32
+                self.logits = synth.device_logits(rows, V, dev, seed=self.seed, std=self.wl.logits_std,
+                                                  boost_max=self.wl.logits_boost, dtype=dt)
+            self.max_prob = torch.empty(rows, dtype=torch.float32, device=dev)
+            self.top1 = torch.empty(rows, dtype=torch.int32, device=dev)
+            self.margin = torch.empty(rows, dtype=torch.float32, device=dev)
+            self.ws = A.scores_workspace(rows, V, dev)
+
+    # ------------------------------------------------------------------ pieces
+    def _timed(self, kind, fn):
+        if not self.time_attention:
+            fn()
+            return
+        s, e = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        s.record()
+        fn()
+        e.record()
+        self.attn_events.append((s, e, kind))
+
+    def _forward(self, refresh: bool, flags):
+        outs = []
+        for layer in range(self.L):
+            if refresh:
+                self._timed("refresh", lambda: A.archer_prompt_refresh(
+                    self.shape, self.q_all[layer], self.k_new[layer], self.v_new[layer], self.k_resp[layer],
+                    self.v_resp[layer], self.out_full, None, self.k_cache[layer], self.v_cache[layer],
+                    refresh_flags=flags))
+                if self.record:
+                    outs.append(self.out_full.clone())
+            else:
+                self._timed("step", lambda: A.archer_attn_step(
+                    self.shape, self.q_resp[layer], self.k_cache[layer], self.v_cache[layer], self.k_resp[layer],
+                    self.v_resp[layer], self.out_step))
+                if self.record:
+                    outs.append(self.out_step.clone())
+        return outs
+
+    def _score(self, t):
+        if not self.score:
+            return None
+        if self.source == "host":
+            z = synth.traj_logits(self.wl, self.seed, t)
+            if self.wl.logits_dtype == "bf16":
+                self.logits = _dev_bits(z, self.device)
+            else:
+                self.logits = torch.from_numpy(z).to(self.device)
+        self._timed("score", lambda: A.archer_decode_scores(self.logits, self.max_prob, self.top1, self.margin,
+                                                            workspace=self.ws))
+        if self.record:
+            return {"max_prob": self.max_prob.clone(), "top1": self.top1.clone(), "margin": self.margin.clone()}
+        return None
+
+    def _stage_redraw(self, t):
+        B, P = self.B, self.P
+        if self.wl.redraws_per_step == 0:
+            return
+        bidx = torch.arange(B, device=self.device)[:, None]
+        if self.source == "host":
+            pos, new = synth.traj_redraw(self.wl, self.seed, t, self.g_host)
+            self.g_host[np.arange(B)[:, None], pos] = new
+            pos_d = torch.from_numpy(pos).to(self.device)
+            self.g[bidx, pos_d] = torch.from_numpy(new).to(self.device)
+            for layer in range(self.L):
+                rows = synth.traj_redraw_rows(self.wl, self.seed, t, layer)
+                q, k, v = (_dev_bits(rows[c], self.device) for c in ("q", "k", "v"))
+                self.q_resp[layer][bidx, pos_d] = q
+                self.q_all[layer][bidx, P + pos_d] = q
+                self.k_resp[layer][bidx, pos_d] = k
+                self.v_resp[layer][bidx, pos_d] = v
+        else:
+            pos_d, new_d = self.plan[(t - 1) % len(self.plan)]
+            self.g[bidx, pos_d] = new_d
+            slot = (t - 1) % self.pool_steps
+            q, k, v = self.pool["q"][slot], self.pool["k"][slot], self.pool["v"][slot]
+            self.q_resp[:, bidx, pos_d] = q
+            self.q_all[:, bidx, P + pos_d] = q
+            self.k_resp[:, bidx, pos_d] = k
+            self.v_resp[:, bidx, pos_d] = v
+
+    def _stage_fresh_prompt(self, t):
+        # Fresh prompt Q/K/V for a refresh (the model's prompt states under g_t).
+        if self.source != "host":
+            return            # device source: the resident fresh-prompt tensors stand in
+        for layer in range(self.L):
+            fp = synth.traj_fresh_prompt(self.wl, self.seed, t, layer)
+            self.q_all[layer][:, :self.P] = _dev_bits(fp["q_prompt"], self.device)
+            self.k_new[layer].copy_(_dev_bits(fp["k_new"], self.device))
+            self.v_new[layer].copy_(_dev_bits(fp["v_new"], self.device))
+
+    # ------------------------------------------------------------------ steps
+    def build(self):
+        """Step 0: FullForward in every layer builds the prompt cache; then score."""
+        self.t = 0
+        self.flag.fill_(1)
+        outs = self._forward(True, None)
+        self.g_anchor.copy_(self.g)
+        self.age.zero_()
+        sc = self._score(0)
+        self.n_refresh_steps = 1
+        return {"t": 0, "flag": np.ones(self.B, np.uint8), "dist": np.zeros(self.B, np.int32), "out": outs,
+                "scores": sc}
+
+    def step(self):
+        t = self.t = self.t + 1
+        self._stage_redraw(t)
+        A.archer_should_refresh(self.g, self.g_anchor, self.age, self.K, self.max_age, True, self.dist, self.flag)
+        self.flag_host.copy_(self.flag, non_blocking=True)
+        torch.cuda.current_stream().synchronize()
+        flags = self.flag_host.numpy()
+        refresh = bool(flags.any())
+        if refresh:
+            self.n_refresh_steps += 1
+            self._stage_fresh_prompt(t)
+        outs = self._forward(refresh, self.flag if refresh else None)
+        sc = self._score(t)
+        rec = {"t": t, "flag": flags.copy(), "out": outs, "scores": sc}
+        if self.record:
+            rec["dist"] = self.dist.cpu().numpy()
+        return rec
+
+    def attention_flops(self, refresh: bool) -> float:
+        """Algorithmic attention FLOPs of one step over all layers: 4 B Hq M N D
+        (Q K^T and P V, 2 flops per multiply-add), M = N on refresh, G cached."""
+        M = self.N if refresh else self.G
+        return 4.0 * self.B * self.Hq * M * self.N * self.D * self.L

@@ -1,0 +1,66 @@
+"""Algorithm 1 end to end on the GPU (through the C ABI) against the oracle's run
+of the same seeded trajectory: refresh flags bit-exact at every step, attention
+outputs of every layer within 2e-2 + 2e-2 |ref|, scores within the scoring
+tolerances (top-1 exact where the oracle margin >= 1e-4)."""
+import numpy as np
+import pytest
+import torch
+
+from oracle import trajectory as OT
+from paper_2608_08086_gb300 import synth
+
+pytestmark = pytest.mark.gpu
+
+MIXED = synth.Workload("mixed", synth.AttnShape(3, 96, 40, 4, 2, 64), layers=2, steps=10, redraws_per_step=3,
+                       radius_k=8, max_age=0, vocab=500, logits_rows=120, logits_dtype="bf16", logits_std=2.0)
+
+
+def _host(t):
+    if t.dtype == torch.bfloat16:
+        return synth.bf16_bits_to_f64(t.view(torch.int16).cpu().numpy().view(np.uint16))
+    return t.double().cpu().numpy()
+
+
+def _compare(wl, mode="archer"):
+    from paper_2608_08086_gb300.trajectory import DeviceTrajectory
+    ref = OT.run(wl, seed=0, mode=mode)
+    tr = DeviceTrajectory(wl, seed=0, mode=mode, source="host", record=True)
+    got = [tr.build()] + [tr.step() for _ in range(wl.steps)]
+    torch.cuda.synchronize()
+    P = wl.shape.prompt_len
+    mixed_seen = False
+    for r, g in zip(ref, got):
+        t = r["t"]
+        np.testing.assert_array_equal(g["flag"], r["flag"], err_msg=f"flags at step {t}")
+        refreshed = bool(r["flag"].any())
+        mixed_seen |= refreshed and not r["flag"].all()
+        for layer, (o_ref, o_got) in enumerate(zip(r["out"], g["out"])):
+            o_got = _host(o_got)
+            if refreshed:
+                for b in range(wl.shape.batch):
+                    sel = slice(None) if r["flag"][b] else slice(P, None)
+                    err = np.abs(o_got[b, sel] - o_ref[b, sel]) - (2e-2 + 2e-2 * np.abs(o_ref[b, sel]))
+                    assert (err <= 0).all(), f"step {t} layer {layer} seq {b}"
+            else:
+                err = np.abs(o_got - o_ref) - (2e-2 + 2e-2 * np.abs(o_ref))
+                assert (err <= 0).all(), f"step {t} layer {layer}"
+        if r["scores"] is not None:
+            s_ref, s_got = r["scores"], {k: v.cpu().numpy() for k, v in g["scores"].items()}
+            keep = s_ref["margin"] >= 1e-4
+            assert (s_got["top1"][keep] == s_ref["top1"][keep]).all(), f"top-1 at step {t}"
+            for k in ("max_prob", "margin"):
+                err = np.abs(s_got[k] - s_ref[k]) - (1e-5 + 1e-4 * np.abs(s_ref[k]))
+                assert (err <= 0).all(), f"{k} at step {t}"
+    return mixed_seen
+
+
+def test_tiny_trajectory_matches_oracle():
+    _compare(synth.WORKLOADS["tiny"])
+
+
+def test_tiny_trajectory_eager_matches_oracle():
+    _compare(synth.WORKLOADS["tiny"], mode="eager")
+
+
+def test_mixed_batch_trajectory_matches_oracle():
+    assert _compare(MIXED), "the workload was chosen to produce mixed per-sequence refresh flags"
