@@ -111,8 +111,9 @@ size_t archer_attn_workspace_size(const archer_shape* shape, int n_queries);
  *   cur_prob = p[cur_tokens[r]] where mask_state[r] == 0 and
  *              0 <= cur_tokens[r] < vocab, else 0   (skipped when NULL)
  *   logits:   [batch * resp_len rows, row_stride elements], dtype bf16 or f32,
- *             row_stride >= vocab; the row stride in bytes must be a multiple
- *             of 16.  -inf entries have probability 0; NaN gives undefined
+ *             row_stride >= vocab (rows whose start is not 16-byte aligned
+ *             are read element-wise, which is slower).  -inf entries have
+ *             probability 0; NaN gives undefined
  *             results.  A row with no finite entry is undefined.
  *   mask_state [rows] uint8 (may be NULL = unmasked); cur_tokens [rows] int32
  *   (may be NULL); outputs [rows] fp32 / int32 device arrays.

@@ -188,9 +188,10 @@ int archer_decode_scores(int batch, int resp_len, int vocab, int dtype, const vo
   if (rows > 0x7FFFFFFFll) { set_error("too many rows"); return ARCHER_ERR_UNSUPPORTED; }
   if (rows == 0) return ARCHER_OK;
   const int esize = dtype == ARCHER_DTYPE_BF16 ? 2 : 4;
-  int st = check_ptrs("logits", {logits});
-  if (st) return st;
-  if ((row_stride * esize) % 16 != 0) { set_error("row stride must be a multiple of 16 bytes"); return ARCHER_ERR_ARG; }
+  if (!logits || (reinterpret_cast<uintptr_t>(logits) % esize) != 0) {
+    set_error("logits is NULL or not aligned to its element size");
+    return ARCHER_ERR_ARG;
+  }
   if (!max_prob || !top1 || !margin) { set_error("max_prob, top1 and margin must not be NULL"); return ARCHER_ERR_ARG; }
   return decode_scores_launch(static_cast<int>(rows), vocab, dtype, logits, row_stride, mask_state, cur_tokens,
                               max_prob, top1, margin, cur_prob, workspace, ws_bytes,

@@ -53,16 +53,16 @@ __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
 
 // Waits for the phase with the given parity to complete.  Gives up (returns
 // false) when *abort is set by another role of the CTA, or after
-// kWaitLimitCycles, in which case it sets *abort and ORs kErrWaitTimeout into
+// `limit` SM clocks, in which case it sets *abort and ORs kErrWaitTimeout into
 // the device error word.
 __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, volatile int* abort,
-                                          int* err_word) {
+                                          int* err_word, long long limit = kWaitLimitCycles) {
   if (mbar_try_wait(bar, parity)) return true;
   const long long t0 = clock64();
   while (true) {
     if (mbar_try_wait(bar, parity)) return true;
     if (*abort) return false;
-    if (clock64() - t0 > kWaitLimitCycles) {
+    if (clock64() - t0 > limit) {
       *abort = 1;
       if (err_word) atomicOr(err_word, kErrWaitTimeout);
       return false;

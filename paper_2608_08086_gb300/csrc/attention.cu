@@ -22,6 +22,7 @@
 
 #include <cmath>
 #include <cstdio>
+#include <cstdlib>
 #include <mutex>
 
 #include <cudaTypedefs.h>
@@ -44,6 +45,8 @@ struct AttnParams {
   int P, G, Hq, Hkv, M;
   int q_begin_refresh, q_begin_cached, default_refresh;
   float scale_log2;           // softmax_scale * log2(e)
+  long long wait_limit;       // SM clocks a bounded wait may take
+  int debug_skip_last_pv;     // test hook: withhold the last PV and its commits
   const uint8_t* flags;
   __nv_bfloat16* out;
   float* lse;
@@ -72,12 +75,12 @@ struct Layout {
 // Warp-uniform bounded wait for the softmax warps (tcgen05.ld/st are
 // .sync.aligned, so all 32 lanes must take the same path).
 __device__ __forceinline__ bool warp_wait(uint32_t bar, uint32_t parity, volatile int* abort,
-                                          int* err) {
+                                          int* err, long long limit) {
   const long long t0 = clock64();
   while (true) {
     const bool done = mbar_try_wait(bar, parity);
     if (__all_sync(0xffffffffu, done)) return true;
-    const bool give_up = (*abort != 0) || (clock64() - t0 > kWaitLimitCycles);
+    const bool give_up = (*abort != 0) || (clock64() - t0 > limit);
     if (__any_sync(0xffffffffu, give_up)) {
       if ((threadIdx.x & 31) == 0 && !*abort) {
         *abort = 1;
@@ -167,14 +170,14 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
         const bool in_prompt = j < n_p;
         const int row = in_prompt ? j * kBN : (j - n_p) * kBN;
         const int ks = j % L::kKS, kuse = j / L::kKS;
-        if (kuse > 0 && !mbar_wait(bar_k_empty + 8 * ks, (kuse - 1) & 1, abort, p.err)) break;
+        if (kuse > 0 && !mbar_wait(bar_k_empty + 8 * ks, (kuse - 1) & 1, abort, p.err, p.wait_limit)) break;
         mbar_arrive_expect_tx(bar_k_full + 8 * ks, L::kTile);
         const CUtensorMap* mk = in_prompt ? mKp : &tmKg;
         for (int c = 0; c < L::kChunks; ++c)
           tma_load_4d(sK + ks * L::kTile + c * kChunkBytes, mk, bar_k_full + 8 * ks, c * 64, kvh,
                       row, b);
         const int vs = j % L::kVS, vuse = j / L::kVS;
-        if (vuse > 0 && !mbar_wait(bar_v_empty + 8 * vs, (vuse - 1) & 1, abort, p.err)) break;
+        if (vuse > 0 && !mbar_wait(bar_v_empty + 8 * vs, (vuse - 1) & 1, abort, p.err, p.wait_limit)) break;
         mbar_arrive_expect_tx(bar_v_full + 8 * vs, L::kTile);
         const CUtensorMap* mv = in_prompt ? mVp : &tmVg;
         for (int c = 0; c < L::kChunks; ++c)
@@ -203,7 +206,7 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
                   idesc_pv, (acc || kk > 0) ? 1u : 0u);
         }
       };
-      bool ok = mbar_wait(bar_q_full, 0, abort, p.err) && mbar_wait(bar_k_full, 0, abort, p.err);
+      bool ok = mbar_wait(bar_q_full, 0, abort, p.err, p.wait_limit) && mbar_wait(bar_k_full, 0, abort, p.err, p.wait_limit);
       if (ok) {
         tc_fence_after();
         issue_qk(kColS0, sK);
@@ -213,7 +216,7 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
       for (int j = 0; ok && j < T; ++j) {
         if (j + 1 < T) {
           const int ks = (j + 1) % L::kKS;
-          if (!mbar_wait(bar_k_full + 8 * ks, ((j + 1) / L::kKS) & 1, abort, p.err)) break;
+          if (!mbar_wait(bar_k_full + 8 * ks, ((j + 1) / L::kKS) & 1, abort, p.err, p.wait_limit)) break;
           tc_fence_after();
           const int sb = (j + 1) & 1;
           issue_qk(sb ? kColS1 : kColS0, sK + ks * L::kTile);
@@ -221,8 +224,9 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
           umma_commit(bar_k_empty + 8 * ks);
         }
         const int vs = j % L::kVS;
-        if (!mbar_wait(bar_v_full + 8 * vs, (j / L::kVS) & 1, abort, p.err)) break;
-        if (!mbar_wait(bar_p_full + 8 * (j & 1), (j >> 1) & 1, abort, p.err)) break;
+        if (!mbar_wait(bar_v_full + 8 * vs, (j / L::kVS) & 1, abort, p.err, p.wait_limit)) break;
+        if (!mbar_wait(bar_p_full + 8 * (j & 1), (j >> 1) & 1, abort, p.err, p.wait_limit)) break;
+        if (p.debug_skip_last_pv && j == T - 1) break;   // the softmax's last wait must now expire
         tc_fence_after();
         issue_pv((j & 1) ? kColP1 : kColP0, sV + vs * L::kTile, j > 0);
         umma_commit(bar_pv_done + 8 * (j & 1));
@@ -240,7 +244,7 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
     bool ok = true;
     for (int j = 0; j < T; ++j) {
       const int sb = j & 1;
-      if (!warp_wait(bar_s_full + 8 * sb, (j >> 1) & 1, abort, p.err)) { ok = false; break; }
+      if (!warp_wait(bar_s_full + 8 * sb, (j >> 1) & 1, abort, p.err, p.wait_limit)) { ok = false; break; }
       tc_fence_after();
       uint32_t sr[128];
       tmem_ld_128(t_lane + (sb ? kColS1 : kColS0), sr);
@@ -266,14 +270,14 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
       // barrier two phases ahead.
       if (j >= 2) {
         // P[sb] was last read by PV_{j-2}.
-        if (!warp_wait(bar_pv_done + 8 * sb, ((j - 2) >> 1) & 1, abort, p.err)) { ok = false; break; }
+        if (!warp_wait(bar_pv_done + 8 * sb, ((j - 2) >> 1) & 1, abort, p.err, p.wait_limit)) { ok = false; break; }
         tc_fence_after();
       }
       if (j == 0) {
         m_used = mt2;
       } else if (__any_sync(0xffffffffu, mt2 > m_used + 8.0f)) {
         // Rescale O: wait until PV_{j-1} has finished accumulating into it.
-        if (!warp_wait(bar_pv_done + 8 * (sb ^ 1), ((j - 1) >> 1) & 1, abort, p.err)) { ok = false; break; }
+        if (!warp_wait(bar_pv_done + 8 * (sb ^ 1), ((j - 1) >> 1) & 1, abort, p.err, p.wait_limit)) { ok = false; break; }
         tc_fence_after();
         const float m_new = fmaxf(m_used, mt2);
         const float alpha = ex2_approx(m_used - m_new);
@@ -303,7 +307,7 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
       tc_fence_before();
       mbar_arrive(bar_p_full + 8 * sb);
     }
-    if (ok && warp_wait(bar_pv_done + 8 * ((T - 1) & 1), ((T - 1) >> 1) & 1, abort, p.err)) {
+    if (ok && warp_wait(bar_pv_done + 8 * ((T - 1) & 1), ((T - 1) >> 1) & 1, abort, p.err, p.wait_limit)) {
       tc_fence_after();
       const float inv_l = 1.0f / l_sum;
       const int q = q0 + r;
@@ -398,6 +402,12 @@ int launch_d(const AttnCall& c, cudaStream_t stream) {
   prm.q_begin_cached = c.q_begin_cached;
   prm.default_refresh = c.default_refresh;
   prm.scale_log2 = c.scale * 1.4426950408889634f;
+  // Test hook (host-set): ARCHER_DEBUG_STALL_ATTENTION=1 withholds the last PV
+  // product, so a bounded wait expires after ~1e6 clocks and the call reports
+  // ARCHER_ERR_TIMEOUT through archer_check_device; the context stays usable.
+  const char* stall = std::getenv("ARCHER_DEBUG_STALL_ATTENTION");
+  prm.debug_skip_last_pv = (stall && stall[0] == '1') ? 1 : 0;
+  prm.wait_limit = prm.debug_skip_last_pv ? 1000000ll : kWaitLimitCycles;
   prm.flags = c.flags;
   prm.out = static_cast<__nv_bfloat16*>(c.out);
   prm.lse = c.lse;

@@ -150,7 +150,8 @@ __global__ void __launch_bounds__(kThreads)
 decode_scores_kernel(const T* __restrict__ logits, int64_t row_stride, int vocab, int chunks,
                      const uint8_t* __restrict__ mask_state, const int32_t* __restrict__ cur_tokens,
                      float* __restrict__ max_prob, int32_t* __restrict__ top1, float* __restrict__ margin,
-                     float* __restrict__ cur_prob, int* __restrict__ counters, Partial* __restrict__ parts) {
+                     float* __restrict__ cur_prob, int* __restrict__ counters, Partial* __restrict__ parts,
+                     int aligned) {
   constexpr int E = Vec<T>::kElems;              // elements per 16-byte word
   constexpr int dtype = sizeof(T) == 2 ? ARCHER_DTYPE_BF16 : ARCHER_DTYPE_F32;
   __shared__ Smem sm;
@@ -165,10 +166,10 @@ decode_scores_kernel(const T* __restrict__ logits, int64_t row_stride, int vocab
 #pragma unroll
   for (int u = 0; u < kUnroll; ++u) {
     const int64_t e0 = chunk_elem0 + (static_cast<int64_t>(u) * kThreads + threadIdx.x) * E;
-    if (e0 + E <= vocab) {
+    if (aligned && e0 + E <= vocab) {
       w[u] = __ldcs(zw + e0 / E);                 // streamed once: evict-first
     } else {
-      // ragged tail: element-wise, -inf past the vocabulary
+      // ragged tail or rows not 16-byte aligned: element-wise, -inf past the vocabulary
       float v[E];
 #pragma unroll
       for (int e = 0; e < E; ++e) v[e] = (e0 + e < vocab) ? load_logit(zrow, dtype, (int)(e0 + e)) : -INFINITY;
@@ -321,6 +322,8 @@ int decode_scores_launch(int rows, int vocab, int dtype, const void* logits, int
     parts = reinterpret_cast<Partial*>(static_cast<char*>(workspace) +
                                        ((static_cast<size_t>(rows) * sizeof(int) + 255) / 256) * 256);
   }
+  const int esize = dtype == ARCHER_DTYPE_BF16 ? 2 : 4;
+  const int aligned = (reinterpret_cast<uintptr_t>(logits) % 16 == 0) && ((row_stride * esize) % 16 == 0);
   const long long grid = static_cast<long long>(rows) * chunks;
   if (grid > 0x7FFFFFFFll) {
     set_error("decode_scores grid too large");
@@ -329,11 +332,11 @@ int decode_scores_launch(int rows, int vocab, int dtype, const void* logits, int
   if (dtype == ARCHER_DTYPE_BF16) {
     decode_scores_kernel<__nv_bfloat16><<<(unsigned)grid, kThreads, 0, stream>>>(
         static_cast<const __nv_bfloat16*>(logits), row_stride, vocab, chunks, mask_state, cur_tokens, max_prob, top1,
-        margin, cur_prob, counters, parts);
+        margin, cur_prob, counters, parts, aligned);
   } else {
     decode_scores_kernel<float><<<(unsigned)grid, kThreads, 0, stream>>>(
         static_cast<const float*>(logits), row_stride, vocab, chunks, mask_state, cur_tokens, max_prob, top1, margin,
-        cur_prob, counters, parts);
+        cur_prob, counters, parts, aligned);
   }
   return cuda_status(cudaGetLastError(), "decode_scores launch");
 }

@@ -74,7 +74,7 @@ def test_bad_scoring_and_rule_arguments_rejected(lib):
         ctypes.c_size_t, ctypes.c_void_p]
     p = ctypes.c_void_p(0x10000)
     assert f(1, 4, 100, 0, p, 50, None, None, p, p, p, None, None, 0, None) == -1     # stride < vocab
-    assert f(1, 4, 100, 0, p, 100, None, None, p, p, p, None, None, 0, None) == -1    # 200 B stride
+    assert f(1, 4, 100, 0, ctypes.c_void_p(0x10001), 100, None, None, p, p, p, None, None, 0, None) == -1  # odd
     assert f(1, 4, 104, 7, p, 104, None, None, p, p, p, None, None, 0, None) == -2    # dtype
     assert f(1, 4, 104, 0, p, 104, None, None, None, p, p, None, None, 0, None) == -1  # null output
     g = lib.archer_should_refresh

@@ -247,6 +247,7 @@ def test_scores_full_scoring_workload_bf16(A):
 
 
 @pytest.mark.parametrize("V,stride,dtype", [(1001, 1008, "bf16"), (1001, 1004, "f32"), (1, 8, "bf16"),
+                                            (1001, 1001, "bf16"), (999, 1001, "f32"),
                                             (17, 20, "f32"), (40000, 40000, "bf16"), (33000, 33004, "f32"),
                                             (152064, 152064, "bf16")])
 def test_scores_ragged_vocab_and_stride(A, V, stride, dtype):
@@ -254,7 +255,8 @@ def test_scores_ragged_vocab_and_stride(A, V, stride, dtype):
     z = synth.logits(rows, V, seed=5, std=2.0, boost_max=3.0, dtype=dtype)
     zf = synth.bf16_bits_to_f64(z) if dtype == "bf16" else z.astype(np.float64)
     zf[3, :] = 0.5                               # constant row: tie everywhere
-    zf[4, ::2] = -np.inf                         # half the vocabulary excluded
+    if V > 2:
+        zf[4, ::2] = -np.inf                     # half the vocabulary excluded
     zf[5, :] = -np.inf
     zf[5, V // 2] = 1.0                          # a single finite entry
     pad = np.full((rows, stride), -np.inf)
