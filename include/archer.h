@@ -128,6 +128,33 @@ int archer_decode_scores(int batch, int resp_len, int vocab, int dtype, const vo
 size_t archer_decode_scores_workspace_size(int rows, int vocab);
 
 /*
+ * Decoder scoring without any device allocation.  The paper has no
+ * counterpart: this serves callers that cannot allocate a workspace -- code
+ * running inside another framework's memory pool, latency-critical loops that
+ * must not pay cudaMalloc's device synchronisation, thin bindings with no
+ * allocator at hand.  Same arguments and results as archer_decode_scores,
+ * without workspace / ws_bytes.
+ *   Scratch: a static device array of ARCHER_NOALLOC_SCRATCH_BYTES (4 MiB),
+ *   created when the library is loaded on a device and held by that device
+ *   until the process exits.  A call needing more
+ *   (archer_decode_scores_workspace_size(rows, vocab) > 4 MiB, e.g. more than
+ *   about 13,000 rows of a 152,064-entry bf16 vocabulary) returns
+ *   ARCHER_ERR_UNSUPPORTED and launches nothing.
+ *   The first call on a device looks up the array's device address (this may
+ *   load the library's device code on that device); make that first call
+ *   before any stream capture.
+ *   Every call shares the one array per device and clears its counters on
+ *   `stream` before launching: calls that can overlap on the GPU (other
+ *   streams, other host threads) race and must be serialised by the caller.
+ *   Calls no cudaMalloc / cudaFree.
+ */
+#define ARCHER_NOALLOC_SCRATCH_BYTES (4u << 20)
+int archer_decode_scores_noalloc(int batch, int resp_len, int vocab, int dtype, const void* logits,
+                                 int64_t row_stride, const uint8_t* mask_state,
+                                 const int32_t* cur_tokens, float* max_prob, int32_t* top1,
+                                 float* margin, float* cur_prob, void* stream);
+
+/*
  * Refresh rule -- Sec. 4.2, Eq. archer-distance and Eq. archer-controller,
  * with the cache-age signal A_t = t - r of Sec. 6 as an optional cap:
  *   age_t   = age[b] + 1           (denoising steps since the anchor, this one included)

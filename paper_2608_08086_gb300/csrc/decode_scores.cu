@@ -17,6 +17,7 @@
 
 #include <cfloat>
 #include <cmath>
+#include <mutex>
 
 #include "archer_device.cuh"
 #include "archer_internal.h"
@@ -342,3 +343,85 @@ int decode_scores_launch(int rows, int vocab, int dtype, const void* logits, int
 }
 
 }  // namespace archer
+
+// ---------------------------------------------------------------------------
+// Scoring without any device allocation.
+//
+// Some callers cannot allocate device memory for the workspace: code that runs
+// inside another framework's memory pool (where a raw cudaMalloc bypasses its
+// accounting), latency-critical loops that must not pay cudaMalloc's implicit
+// device synchronisation, and thin foreign-function bindings with no allocator
+// at hand.  For them the chunk partials and ticket counters live in this
+// file-scope array, created when the library is loaded on a device and held
+// by every GPU that loads the library until the process exits.
+// ---------------------------------------------------------------------------
+namespace archer {
+namespace {
+
+constexpr size_t kNoAllocScratchBytes = ARCHER_NOALLOC_SCRATCH_BYTES;
+static __device__ __align__(256) unsigned char g_scores_scratch[kNoAllocScratchBytes];
+
+// Device address of g_scores_scratch on the current device.  Host code cannot
+// use the array's name as a device pointer (it is a host-side stand-in), so the
+// address is looked up once per device, with that device current.
+int scratch_address(void** out) {
+  static void* addr[64] = {nullptr};
+  static std::mutex mu;
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return cuda_status(e, "cudaGetDevice");
+  if (dev < 0 || dev >= 64) {
+    set_error("device ordinal %d out of range", dev);
+    return ARCHER_ERR_UNSUPPORTED;
+  }
+  std::lock_guard<std::mutex> lock(mu);
+  if (!addr[dev]) {
+    void* p = nullptr;
+    e = cudaGetSymbolAddress(&p, g_scores_scratch);
+    if (e != cudaSuccess) return cuda_status(e, "cudaGetSymbolAddress(scoring scratch)");
+    addr[dev] = p;
+  }
+  *out = addr[dev];
+  return ARCHER_OK;
+}
+
+}  // namespace
+}  // namespace archer
+
+extern "C" int archer_decode_scores_noalloc(int batch, int resp_len, int vocab, int dtype, const void* logits,
+                                            int64_t row_stride, const uint8_t* mask_state,
+                                            const int32_t* cur_tokens, float* max_prob, int32_t* top1,
+                                            float* margin, float* cur_prob, void* stream) {
+  using namespace archer;
+  if (batch < 0 || resp_len < 0 || vocab < 1 || row_stride < vocab) {
+    set_error("bad scoring shape: batch=%d resp_len=%d vocab=%d row_stride=%lld", batch, resp_len, vocab,
+              (long long)row_stride);
+    return ARCHER_ERR_ARG;
+  }
+  const long long rows = static_cast<long long>(batch) * resp_len;
+  if (rows > 0x7FFFFFFFll) {
+    set_error("too many rows");
+    return ARCHER_ERR_UNSUPPORTED;
+  }
+  if (rows == 0) return ARCHER_OK;
+  const size_t need = decode_scores_ws_bytes(static_cast<int>(rows), vocab);
+  if (need > kNoAllocScratchBytes) {
+    set_error("%lld rows of %d logits need %zu bytes of scoring scratch; the allocation-free entry point has "
+              "%zu (use archer_decode_scores with a workspace)",
+              rows, vocab, need, kNoAllocScratchBytes);
+    return ARCHER_ERR_UNSUPPORTED;
+  }
+  void* scratch = nullptr;
+  int st = scratch_address(&scratch);
+  if (st) return st;
+  const cudaStream_t s = static_cast<cudaStream_t>(stream);
+  if (need > 0) {
+    // The ticket counters must start at zero; a call normally leaves them so,
+    // but clear them in case an earlier call on this device did not finish.
+    const size_t counter_bytes = ((static_cast<size_t>(rows) * sizeof(int) + 255) / 256) * 256;
+    cudaError_t e = cudaMemsetAsync(scratch, 0, counter_bytes, s);
+    if (e != cudaSuccess) return cuda_status(e, "clearing the scoring scratch counters");
+  }
+  return archer_decode_scores(batch, resp_len, vocab, dtype, logits, row_stride, mask_state, cur_tokens, max_prob,
+                              top1, margin, cur_prob, scratch, kNoAllocScratchBytes, stream);
+}
