@@ -8,16 +8,26 @@
 // response segment through two TMA tensor maps, so the concatenation is never
 // formed in memory.  GQA: query head h reads KV head h / (Hq / Hkv).
 //
-// One CTA = one 128-row query tile of one (b, h); 6 warps:
-//   warps 0-3  softmax: thread t owns query row t (TMEM lane t); online
-//              softmax in the log2 domain with a lazily raised running max
-//              (O and l are rescaled only when the tile max exceeds the max in
-//              use by more than 2^8), P written to TMEM as bf16 pairs.
-//   warp 4     TMA producer: Q once, then K and V tiles into 2-stage rings.
-//   warp 5     MMA issuer (one thread): S = Q K^T (SS, K-major operands) into
-//              a double-buffered TMEM S, then O += P V (P from TMEM, V as an
-//              MN-major smem operand), fp32 accumulation in TMEM.
-// TMEM (512 columns): S0 [0,128) S1 [128,256) O [256,256+D) P0 [384,448) P1 [448,512).
+// One CTA = two 128-row query tiles (A and B) of one (b, h) sharing every K/V
+// tile; 10 warps:
+//   warps 0-3  softmax of tile A, warps 4-7 softmax of tile B: thread t of a
+//              warpgroup owns query row t (TMEM lane t).  S is read in two
+//              64-column halves; exponentials use the running max in use and
+//              the max is raised lazily (only when a half's max exceeds it by
+//              more than 2^8), rescaling l and O.  Each half of P (bf16 pairs)
+//              is written over S's own TMEM columns and handed to the MMA warp
+//              at once, so P V of the first half overlaps the second half's
+//              exponentials.
+//   warp 8     TMA producer: Q_A, Q_B once, then K tiles (3-stage ring) and V
+//              tiles (2-stage ring) of 128 keys.
+//   warp 9     MMA issuer (one thread), per K/V tile j:
+//                PV_A(j) in two halves, QK_A(j+1), PV_B(j) in two halves, QK_B(j+1)
+//              so the tensor pipe works on one tile while the other tile's
+//              softmax runs.  tcgen05.mma executes in issue order, so QK_X(j+1)
+//              overwrites S_X only after PV_X(j) has read P_X(j), and the commit
+//              that announces S_X(j+1) also covers PV_X(j): when the softmax sees
+//              S_X(j+1), O_X is stable and may be rescaled without a wait.
+// TMEM (512 columns): S_A [0,128) S_B [128,256) O_A [256,256+D) O_B [384,384+D).
 // Every hand-off is an mbarrier; every wait is bounded (archer_device.cuh).
 
 #include <cmath>
@@ -34,11 +44,14 @@
 namespace archer {
 namespace {
 
-constexpr int kBM = 128;          // query rows per CTA (tcgen05 M)
+constexpr int kBM = 128;          // query rows per tile (tcgen05 M)
 constexpr int kBN = 128;          // keys per KV tile (N of Q K^T, K of P V)
-constexpr int kThreads = 192;
+constexpr int kThreads = 320;     // 2 softmax warpgroups + producer warp + MMA warp
+constexpr int kWarpProducer = 8, kWarpMma = 9;
 constexpr uint32_t kTmemCols = 512;
-constexpr uint32_t kColS0 = 0, kColS1 = 128, kColO = 256, kColP0 = 384, kColP1 = 448;
+// TMEM columns of tile t's S (P is written over its first 64 columns) and O.
+__host__ __device__ constexpr uint32_t col_s(int t) { return 128u * static_cast<uint32_t>(t); }
+__host__ __device__ constexpr uint32_t col_o(int t) { return 256u + 128u * static_cast<uint32_t>(t); }
 constexpr uint32_t kChunkBytes = 128 * 128;   // 128 rows x 128 B (64 bf16) swizzle region
 
 struct AttnParams {
@@ -55,21 +68,23 @@ struct AttnParams {
 
 template <int D>
 struct Layout {
-  static constexpr int kChunks = D / 64;                  // 128-byte column chunks
+  static constexpr int kChunks = D / 64;                    // 128-byte column chunks
   static constexpr uint32_t kTile = kChunks * kChunkBytes;  // one 128-row tile of D bf16
-  static constexpr int kKS = 2, kVS = 2;                  // K / V ring stages
-  static constexpr uint32_t kOffQ = 0;
-  static constexpr uint32_t kOffK = kOffQ + kTile;
+  static constexpr int kKS = 3, kVS = 2;                    // K / V ring stages
+  static constexpr uint32_t kOffQ = 0;                      // Q_A, Q_B
+  static constexpr uint32_t kOffK = kOffQ + 2 * kTile;
   static constexpr uint32_t kOffV = kOffK + kKS * kTile;
   static constexpr uint32_t kOffBar = kOffV + kVS * kTile;
-  // q_full, k_full[KS], k_empty[KS], v_full[VS], v_empty[VS], s_full[2], p_full[2], pv_done[2]
-  static constexpr int kBars = 1 + 2 * kKS + 2 * kVS + 2 + 2 + 2;
+  // q_full, k_full[KS], k_empty[KS], v_full[VS], v_empty[VS],
+  // s_full[2], p_half0[2], p_half1[2], pv_half0_done[2]
+  static constexpr int kBars = 1 + 2 * kKS + 2 * kVS + 8;
   static constexpr uint32_t kOffHolder = kOffBar + 8 * kBars;
   static constexpr uint32_t kOffAbort = kOffHolder + 4;
   static constexpr uint32_t kUsed = kOffAbort + 4;
   // + 1 KB to align the base to 1024 B; at least 120 KB so that one CTA
   // holds an SM (the CTA allocates all 512 TMEM columns).
   static constexpr uint32_t kSmemBytes = (kUsed + 1024 > 120 * 1024) ? kUsed + 1024 : 120 * 1024;
+  static_assert(kUsed + 1024 <= 232448, "shared memory budget");
 };
 
 // Warp-uniform bounded wait for the softmax warps (tcgen05.ld/st are
@@ -91,6 +106,52 @@ __device__ __forceinline__ bool warp_wait(uint32_t bar, uint32_t parity, volatil
   }
 }
 
+__device__ __forceinline__ float max3f(float a, float b, float c) {
+  float d;
+  asm("max.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));
+  return d;
+}
+
+__device__ __forceinline__ float max64(const float (&x)[64]) {
+  float m[4] = {x[0], x[1], x[2], x[3]};
+#pragma unroll
+  for (int c = 4; c < 64; c += 2) m[(c >> 1) & 3] = max3f(m[(c >> 1) & 3], x[c], x[c + 1]);
+  return max3f(m[0], m[1], fmaxf(m[2], m[3]));
+}
+
+// Packed fp32 pairs (two lanes per instruction).
+__device__ __forceinline__ float2 ffma2(float2 a, float2 b, float2 c) {
+  float2 d;
+  asm("{\n\t.reg .b64 ra, rb, rc, rd;\n\t"
+      "mov.b64 ra, {%2, %3};\n\tmov.b64 rb, {%4, %5};\n\tmov.b64 rc, {%6, %7};\n\t"
+      "fma.rn.f32x2 rd, ra, rb, rc;\n\tmov.b64 {%0, %1}, rd;\n}"
+      : "=f"(d.x), "=f"(d.y)
+      : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y), "f"(c.x), "f"(c.y));
+  return d;
+}
+__device__ __forceinline__ float2 fadd2(float2 a, float2 b) {
+  float2 d;
+  asm("{\n\t.reg .b64 ra, rb, rd;\n\t"
+      "mov.b64 ra, {%2, %3};\n\tmov.b64 rb, {%4, %5};\n\t"
+      "add.rn.f32x2 rd, ra, rb;\n\tmov.b64 {%0, %1}, rd;\n}"
+      : "=f"(d.x), "=f"(d.y)
+      : "f"(a.x), "f"(a.y), "f"(b.x), "f"(b.y));
+  return d;
+}
+
+// Loads 64 score columns [c0, c0 + 64) of this lane and masks keys >= valid.
+__device__ __forceinline__ void load_scores(uint32_t taddr, int c0, int valid, float (&x)[64]) {
+  uint32_t r[64];
+  tmem_ld_64(taddr, r);
+#pragma unroll
+  for (int c = 0; c < 64; ++c) x[c] = __uint_as_float(r[c]);
+  if (valid < c0 + 64) {            // only the last tile of a segment is ragged
+#pragma unroll
+    for (int c = 0; c < 64; ++c)
+      if (c0 + c >= valid) x[c] = -INFINITY;
+  }
+}
+
 template <int D>
 __global__ void __launch_bounds__(kThreads, 1)
 attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
@@ -101,10 +162,11 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
   using L = Layout<D>;
   extern __shared__ uint8_t smem_raw[];
 
-  const int qt = blockIdx.x, h = blockIdx.y, b = blockIdx.z;
+  const int tp = blockIdx.x, h = blockIdx.y, b = blockIdx.z;
   const bool refresh = p.flags ? (p.flags[b] != 0) : (p.default_refresh != 0);
-  const int q0 = (refresh ? p.q_begin_refresh : p.q_begin_cached) + qt * kBM;
+  const int q0 = (refresh ? p.q_begin_refresh : p.q_begin_cached) + tp * 2 * kBM;
   if (q0 >= p.M) return;  // uniform over the CTA, before any barrier or TMEM use
+  const bool has_b = q0 + kBM < p.M;
 
   const int kvh = h / (p.Hq / p.Hkv);
   const int n_p = (p.P + kBN - 1) / kBN;
@@ -123,9 +185,10 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
   const uint32_t bar_k_empty = bar_k_full + 8 * L::kKS;
   const uint32_t bar_v_full = bar_k_empty + 8 * L::kKS;
   const uint32_t bar_v_empty = bar_v_full + 8 * L::kVS;
-  const uint32_t bar_s_full = bar_v_empty + 8 * L::kVS;         // + 8 * buffer
-  const uint32_t bar_p_full = bar_s_full + 16;
-  const uint32_t bar_pv_done = bar_p_full + 16;                 // + 8 * (tile & 1)
+  const uint32_t bar_s_full = bar_v_empty + 8 * L::kVS;         // + 8 * tile (A = 0, B = 1)
+  const uint32_t bar_p_h0 = bar_s_full + 16;                    // + 8 * tile: first half of P written
+  const uint32_t bar_p_h1 = bar_p_h0 + 16;                      // + 8 * tile: second half of P written
+  const uint32_t bar_pv_h0 = bar_p_h1 + 16;                     // + 8 * tile: P V of the first half done
   uint32_t* holder = reinterpret_cast<uint32_t*>(gbase + L::kOffHolder);
   volatile int* abort = reinterpret_cast<volatile int*>(gbase + L::kOffAbort);
 
@@ -142,13 +205,14 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
     }
     for (int i = 0; i < 2; ++i) {
       mbar_init(bar_s_full + 8 * i, 1);
-      mbar_init(bar_p_full + 8 * i, kBM);
-      mbar_init(bar_pv_done + 8 * i, 1);
+      mbar_init(bar_p_h0 + 8 * i, kBM);
+      mbar_init(bar_p_h1 + 8 * i, kBM);
+      mbar_init(bar_pv_h0 + 8 * i, 1);
     }
     *abort = 0;
     mbar_fence_init();
   }
-  if (warp == 5) {
+  if (warp == kWarpMma) {
     tmem_alloc(smem_u32(holder), kTmemCols);
     tmem_relinquish();
   }
@@ -157,15 +221,16 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
   tc_fence_after();
   const uint32_t tmem = *holder;
 
-  if (warp == 4) {
+  if (warp == kWarpProducer) {
     // ------------------------------------------------------------ producer
     if (elect_lane0()) {
       const CUtensorMap* mKp = refresh ? &tmKpR : &tmKpC;
       const CUtensorMap* mVp = refresh ? &tmVpR : &tmVpC;
       tma_prefetch_map(&tmQ);
-      mbar_arrive_expect_tx(bar_q_full, L::kTile);
-      for (int c = 0; c < L::kChunks; ++c)
-        tma_load_4d(sQ + c * kChunkBytes, &tmQ, bar_q_full, c * 64, h, q0, b);
+      mbar_arrive_expect_tx(bar_q_full, has_b ? 2 * L::kTile : L::kTile);
+      for (int t = 0; t < (has_b ? 2 : 1); ++t)
+        for (int c = 0; c < L::kChunks; ++c)
+          tma_load_4d(sQ + t * L::kTile + c * kChunkBytes, &tmQ, bar_q_full, c * 64, h, q0 + t * kBM, b);
       for (int j = 0; j < T; ++j) {
         const bool in_prompt = j < n_p;
         const int row = in_prompt ? j * kBN : (j - n_p) * kBN;
@@ -174,167 +239,184 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
         mbar_arrive_expect_tx(bar_k_full + 8 * ks, L::kTile);
         const CUtensorMap* mk = in_prompt ? mKp : &tmKg;
         for (int c = 0; c < L::kChunks; ++c)
-          tma_load_4d(sK + ks * L::kTile + c * kChunkBytes, mk, bar_k_full + 8 * ks, c * 64, kvh,
-                      row, b);
+          tma_load_4d(sK + ks * L::kTile + c * kChunkBytes, mk, bar_k_full + 8 * ks, c * 64, kvh, row, b);
         const int vs = j % L::kVS, vuse = j / L::kVS;
         if (vuse > 0 && !mbar_wait(bar_v_empty + 8 * vs, (vuse - 1) & 1, abort, p.err, p.wait_limit)) break;
         mbar_arrive_expect_tx(bar_v_full + 8 * vs, L::kTile);
         const CUtensorMap* mv = in_prompt ? mVp : &tmVg;
         for (int c = 0; c < L::kChunks; ++c)
-          tma_load_4d(sV + vs * L::kTile + c * kChunkBytes, mv, bar_v_full + 8 * vs, c * 64, kvh,
-                      row, b);
+          tma_load_4d(sV + vs * L::kTile + c * kChunkBytes, mv, bar_v_full + 8 * vs, c * 64, kvh, row, b);
       }
     }
     __syncwarp();
-  } else if (warp == 5) {
+  } else if (warp == kWarpMma) {
     // ------------------------------------------------------------ MMA issuer
     if (elect_lane0()) {
       constexpr uint32_t idesc_qk = idesc_bf16_f32(kBM, kBN, 0, 0);
       constexpr uint32_t idesc_pv = idesc_bf16_f32(kBM, D, 0, 1);
-      auto issue_qk = [&](uint32_t s_col, uint32_t k_tile) {
+      const int n_tiles = has_b ? 2 : 1;
+      auto issue_qk = [&](int t, uint32_t k_tile) {
+        const uint32_t q_tile = sQ + t * L::kTile;
 #pragma unroll
         for (int kk = 0; kk < D / 16; ++kk) {
           const uint32_t off = (kk >> 2) * kChunkBytes + (kk & 3) * 32;
-          umma_ss(tmem + s_col, sdesc_sw128(sQ + off, 16, 1024), sdesc_sw128(k_tile + off, 16, 1024),
+          umma_ss(tmem + col_s(t), sdesc_sw128(q_tile + off, 16, 1024), sdesc_sw128(k_tile + off, 16, 1024),
                   idesc_qk, kk > 0 ? 1u : 0u);
         }
       };
-      auto issue_pv = [&](uint32_t p_col, uint32_t v_tile, bool acc) {
+      // P V over keys [64 * half, 64 * half + 64) of the tile (4 MMAs of K = 16).
+      auto issue_pv = [&](int t, int half, uint32_t v_tile, bool acc) {
 #pragma unroll
-        for (int kk = 0; kk < kBN / 16; ++kk) {
-          umma_ts(tmem + kColO, tmem + p_col + kk * 8, sdesc_sw128(v_tile + kk * 2048, kChunkBytes, 1024),
+        for (int k4 = 0; k4 < 4; ++k4) {
+          const int kk = 4 * half + k4;
+          umma_ts(tmem + col_o(t), tmem + col_s(t) + kk * 8, sdesc_sw128(v_tile + kk * 2048, kChunkBytes, 1024),
                   idesc_pv, (acc || kk > 0) ? 1u : 0u);
         }
       };
-      bool ok = mbar_wait(bar_q_full, 0, abort, p.err, p.wait_limit) && mbar_wait(bar_k_full, 0, abort, p.err, p.wait_limit);
+      bool ok = mbar_wait(bar_q_full, 0, abort, p.err, p.wait_limit) &&
+                mbar_wait(bar_k_full, 0, abort, p.err, p.wait_limit);
       if (ok) {
         tc_fence_after();
-        issue_qk(kColS0, sK);
-        umma_commit(bar_s_full);
+        for (int t = 0; t < n_tiles; ++t) {
+          issue_qk(t, sK);
+          umma_commit(bar_s_full + 8 * t);
+        }
         umma_commit(bar_k_empty);
       }
       for (int j = 0; ok && j < T; ++j) {
-        if (j + 1 < T) {
-          const int ks = (j + 1) % L::kKS;
-          if (!mbar_wait(bar_k_full + 8 * ks, ((j + 1) / L::kKS) & 1, abort, p.err, p.wait_limit)) break;
-          tc_fence_after();
-          const int sb = (j + 1) & 1;
-          issue_qk(sb ? kColS1 : kColS0, sK + ks * L::kTile);
-          umma_commit(bar_s_full + 8 * sb);
-          umma_commit(bar_k_empty + 8 * ks);
-        }
         const int vs = j % L::kVS;
+        const bool more = j + 1 < T;
+        const int ks = (j + 1) % L::kKS;
         if (!mbar_wait(bar_v_full + 8 * vs, (j / L::kVS) & 1, abort, p.err, p.wait_limit)) break;
-        if (!mbar_wait(bar_p_full + 8 * (j & 1), (j >> 1) & 1, abort, p.err, p.wait_limit)) break;
-        if (p.debug_skip_last_pv && j == T - 1) break;   // the softmax's last wait must now expire
-        tc_fence_after();
-        issue_pv((j & 1) ? kColP1 : kColP0, sV + vs * L::kTile, j > 0);
-        umma_commit(bar_pv_done + 8 * (j & 1));
+        for (int t = 0; t < n_tiles; ++t) {
+          if (!mbar_wait(bar_p_h0 + 8 * t, j & 1, abort, p.err, p.wait_limit)) { ok = false; break; }
+          if (p.debug_skip_last_pv && !more) { ok = false; break; }   // the softmax's final wait must expire
+          tc_fence_after();
+          issue_pv(t, 0, sV + vs * L::kTile, j > 0);
+          umma_commit(bar_pv_h0 + 8 * t);
+          if (!mbar_wait(bar_p_h1 + 8 * t, j & 1, abort, p.err, p.wait_limit)) { ok = false; break; }
+          tc_fence_after();
+          issue_pv(t, 1, sV + vs * L::kTile, true);
+          if (more) {
+            if (t == 0 && !mbar_wait(bar_k_full + 8 * ks, ((j + 1) / L::kKS) & 1, abort, p.err, p.wait_limit)) {
+              ok = false;
+              break;
+            }
+            tc_fence_after();
+            issue_qk(t, sK + ks * L::kTile);
+          }
+          umma_commit(bar_s_full + 8 * t);   // S_t(j+1) ready -- or, after the last tile, O_t final
+        }
+        if (!ok) break;
         umma_commit(bar_v_empty + 8 * vs);
+        if (more) umma_commit(bar_k_empty + 8 * ks);
       }
     }
     __syncwarp();
   } else {
     // ------------------------------------------------------------ softmax
-    const int r = threadIdx.x;                                    // query row in the tile
-    const uint32_t t_lane = tmem + (static_cast<uint32_t>(warp * 32) << 16);
-    const float sl2 = p.scale_log2;
-    float m_used = -INFINITY;                                    // running max (log2 units)
-    float l_sum = 0.f;
-    bool ok = true;
-    for (int j = 0; j < T; ++j) {
-      const int sb = j & 1;
-      if (!warp_wait(bar_s_full + 8 * sb, (j >> 1) & 1, abort, p.err, p.wait_limit)) { ok = false; break; }
-      tc_fence_after();
-      uint32_t sr[128];
-      tmem_ld_128(t_lane + (sb ? kColS1 : kColS0), sr);
-      float x[128];
-#pragma unroll
-      for (int c = 0; c < 128; ++c) x[c] = __uint_as_float(sr[c]);
-      const int valid = j < n_p ? min(kBN, p.P - j * kBN) : min(kBN, p.G - (j - n_p) * kBN);
-      if (valid < kBN) {
-#pragma unroll
-        for (int c = 0; c < 128; ++c)
-          if (c >= valid) x[c] = -INFINITY;
-      }
-      float mx[8];
-#pragma unroll
-      for (int i = 0; i < 8; ++i) mx[i] = x[i];
-#pragma unroll
-      for (int c = 8; c < 128; ++c) mx[c & 7] = fmaxf(mx[c & 7], x[c]);
-      const float tmax = fmaxf(fmaxf(fmaxf(mx[0], mx[1]), fmaxf(mx[2], mx[3])),
-                               fmaxf(fmaxf(mx[4], mx[5]), fmaxf(mx[6], mx[7])));
-      const float mt2 = tmax * sl2;
-      // PV_j commits to pv_done[j & 1], so each barrier's next phase belongs to
-      // a PV that needs this thread's next P: no wait below can see its
-      // barrier two phases ahead.
-      if (j >= 2) {
-        // P[sb] was last read by PV_{j-2}.
-        if (!warp_wait(bar_pv_done + 8 * sb, ((j - 2) >> 1) & 1, abort, p.err, p.wait_limit)) { ok = false; break; }
-        tc_fence_after();
-      }
-      if (j == 0) {
-        m_used = mt2;
-      } else if (__any_sync(0xffffffffu, mt2 > m_used + 8.0f)) {
-        // Rescale O: wait until PV_{j-1} has finished accumulating into it.
-        if (!warp_wait(bar_pv_done + 8 * (sb ^ 1), ((j - 1) >> 1) & 1, abort, p.err, p.wait_limit)) { ok = false; break; }
-        tc_fence_after();
-        const float m_new = fmaxf(m_used, mt2);
-        const float alpha = ex2_approx(m_used - m_new);
-        m_used = m_new;
-        l_sum *= alpha;
+    const int t = warp >> 2;                                      // 0 = tile A, 1 = tile B
+    if (t == 0 || has_b) {
+      const int r = threadIdx.x & 127;                            // query row in the tile
+      const uint32_t t_lane = tmem + (static_cast<uint32_t>((warp & 3) * 32) << 16);
+      const uint32_t colS = col_s(t), colO = col_o(t);
+      const uint32_t bar_s = bar_s_full + 8 * t;
+      const uint32_t bar_ph0 = bar_p_h0 + 8 * t, bar_ph1 = bar_p_h1 + 8 * t, bar_pvh0 = bar_pv_h0 + 8 * t;
+      const float sl2 = p.scale_log2;
+      float m_used = -INFINITY;                                  // running max in use (log2 units)
+      float2 l2 = make_float2(0.f, 0.f);                         // row sum, two partial lanes
+      bool ok = true;
+      // O *= a (all 32-bit columns of this lane's O row)
+      auto rescale_o = [&](float a) {
 #pragma unroll
         for (int c0 = 0; c0 < D; c0 += 32) {
           uint32_t o[32];
-          tmem_ld_32(t_lane + kColO + c0, o);
+          tmem_ld_32(t_lane + colO + c0, o);
 #pragma unroll
-          for (int c = 0; c < 32; ++c) o[c] = __float_as_uint(__uint_as_float(o[c]) * alpha);
-          tmem_st_32(t_lane + kColO + c0, o);
+          for (int c = 0; c < 32; ++c) o[c] = __float_as_uint(__uint_as_float(o[c]) * a);
+          tmem_st_32(t_lane + colO + c0, o);
         }
-      }
-      const float neg_m = -m_used;
-      uint32_t pk[64];
-      float ls[4] = {0.f, 0.f, 0.f, 0.f};
-#pragma unroll
-      for (int c = 0; c < 64; ++c) {
-        const float p0 = ex2_approx(fmaf(x[2 * c], sl2, neg_m));
-        const float p1 = ex2_approx(fmaf(x[2 * c + 1], sl2, neg_m));
-        ls[c & 3] += p0 + p1;
-        pk[c] = pack_bf16x2(p0, p1);
-      }
-      l_sum += (ls[0] + ls[1]) + (ls[2] + ls[3]);
-      tmem_st_64(t_lane + (sb ? kColP1 : kColP0), pk);
-      tc_fence_before();
-      mbar_arrive(bar_p_full + 8 * sb);
-    }
-    if (ok && warp_wait(bar_pv_done + 8 * ((T - 1) & 1), ((T - 1) >> 1) & 1, abort, p.err, p.wait_limit)) {
-      tc_fence_after();
-      const float inv_l = 1.0f / l_sum;
-      const int q = q0 + r;
-      const bool live = q < p.M;
-      __nv_bfloat16* orow = p.out + ((static_cast<size_t>(b) * p.M + q) * p.Hq + h) * D;
-#pragma unroll
-      for (int c0 = 0; c0 < D; c0 += 32) {
-        uint32_t o[32];
-        tmem_ld_32(t_lane + kColO + c0, o);
-        uint32_t w[16];
-#pragma unroll
-        for (int c = 0; c < 16; ++c)
-          w[c] = pack_bf16x2(__uint_as_float(o[2 * c]) * inv_l, __uint_as_float(o[2 * c + 1]) * inv_l);
-        if (live) {
-          uint4* dst = reinterpret_cast<uint4*>(orow + c0);
-#pragma unroll
-          for (int v = 0; v < 4; ++v) dst[v] = make_uint4(w[4 * v], w[4 * v + 1], w[4 * v + 2], w[4 * v + 3]);
+      };
+      for (int j = 0; j < T; ++j) {
+        if (!warp_wait(bar_s, j & 1, abort, p.err, p.wait_limit)) { ok = false; break; }
+        tc_fence_after();
+        const int valid = j < n_p ? min(kBN, p.P - j * kBN) : min(kBN, p.G - (j - n_p) * kBN);
+        float x[64];
+        if (j == 0) {
+          load_scores(t_lane + colS, 0, valid, x);
+          float mt = max64(x);
+          load_scores(t_lane + colS + 64, 64, valid, x);
+          mt = fmaxf(mt, max64(x));
+          m_used = mt * sl2;
         }
+#pragma unroll
+        for (int half = 0; half < 2; ++half) {
+          load_scores(t_lane + colS + 64 * half, 64 * half, valid, x);
+          const float hm = max64(x) * sl2;
+          if (__any_sync(0xffffffffu, hm > m_used + 8.0f)) {
+            const float m_new = fmaxf(m_used, hm);
+            const float a = ex2_approx(m_used - m_new);
+            m_used = m_new;
+            l2.x *= a;
+            l2.y *= a;
+            if (half == 1) {
+              // P V of the first half may already have accumulated into O with
+              // the old max: rescale O once it has.
+              if (!warp_wait(bar_pvh0, j & 1, abort, p.err, p.wait_limit)) { ok = false; break; }
+              tc_fence_after();
+            }
+            // (half 0: O holds P V up to tile j-1, complete -- S(j) was announced after it)
+            rescale_o(a);
+          }
+          const float2 neg_m = make_float2(-m_used, -m_used);
+          const float2 slv = make_float2(sl2, sl2);
+          uint32_t pk[32];
+          float2 acc[2] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
+#pragma unroll
+          for (int c = 0; c < 32; ++c) {
+            const float2 y = ffma2(make_float2(x[2 * c], x[2 * c + 1]), slv, neg_m);
+            const float p0 = ex2_approx(y.x);
+            const float p1 = ex2_approx(y.y);
+            acc[c & 1] = fadd2(acc[c & 1], make_float2(p0, p1));
+            pk[c] = pack_bf16x2(p0, p1);
+          }
+          l2 = fadd2(l2, fadd2(acc[0], acc[1]));
+          tmem_st_32(t_lane + colS + 32 * half, pk);     // P half over S columns already read
+          tc_fence_before();
+          mbar_arrive(half == 0 ? bar_ph0 : bar_ph1);
+        }
+        if (!ok) break;
       }
-      if (live && p.lse)
-        p.lse[(static_cast<size_t>(b) * p.Hq + h) * p.M + q] = (m_used + log2f(l_sum)) * 0.69314718055994531f;
+      const float l_sum = l2.x + l2.y;
+      if (ok && warp_wait(bar_s, T & 1, abort, p.err, p.wait_limit)) {
+        tc_fence_after();
+        const float inv_l = 1.0f / l_sum;
+        const int q = q0 + t * kBM + r;
+        const bool live = q < p.M;
+        __nv_bfloat16* orow = p.out + ((static_cast<size_t>(b) * p.M + q) * p.Hq + h) * D;
+#pragma unroll
+        for (int c0 = 0; c0 < D; c0 += 32) {
+          uint32_t o[32];
+          tmem_ld_32(t_lane + colO + c0, o);
+          uint32_t w[16];
+#pragma unroll
+          for (int c = 0; c < 16; ++c)
+            w[c] = pack_bf16x2(__uint_as_float(o[2 * c]) * inv_l, __uint_as_float(o[2 * c + 1]) * inv_l);
+          if (live) {
+            uint4* dst = reinterpret_cast<uint4*>(orow + c0);
+#pragma unroll
+            for (int v = 0; v < 4; ++v) dst[v] = make_uint4(w[4 * v], w[4 * v + 1], w[4 * v + 2], w[4 * v + 3]);
+          }
+        }
+        if (live && p.lse)
+          p.lse[(static_cast<size_t>(b) * p.Hq + h) * p.M + q] = (m_used + log2f(l_sum)) * 0.69314718055994531f;
+      }
     }
   }
 
   tc_fence_before();
   __syncthreads();
-  if (warp == 5) {
+  if (warp == kWarpMma) {
     __syncwarp();
     tc_fence_after();
     tmem_dealloc(tmem, kTmemCols);
@@ -414,7 +496,7 @@ int launch_d(const AttnCall& c, cudaStream_t stream) {
   prm.err = device_error_word();
   // Query tiles needed by the longest query range (a refreshed sequence's).
   const int rows = c.M - (c.flags || c.default_refresh ? c.q_begin_refresh : c.q_begin_cached);
-  const dim3 grid((rows + kBM - 1) / kBM, c.Hq, c.B);
+  const dim3 grid((rows + 2 * kBM - 1) / (2 * kBM), c.Hq, c.B);
   attn_fwd_kernel<D><<<grid, kThreads, L::kSmemBytes, stream>>>(mq, mkr, mvr, mkc, mvc, mkg, mvg, prm);
   return cuda_status(cudaGetLastError(), "attention launch");
 }
