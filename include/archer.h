@@ -117,8 +117,10 @@ size_t archer_attn_workspace_size(const archer_shape* shape, int n_queries);
  *             results.  A row with no finite entry is undefined.
  *   mask_state [rows] uint8 (may be NULL = unmasked); cur_tokens [rows] int32
  *   (may be NULL); outputs [rows] fp32 / int32 device arrays.
- *   workspace: at least archer_decode_scores_workspace_size(rows, vocab) bytes,
- *   zero-filled before its first use; every call leaves it zero-filled again.
+ *   workspace: at least archer_decode_scores_workspace_size(rows, vocab) bytes
+ *   of scratch (chunk partials), any contents; 0 bytes when the vocabulary
+ *   fits one chunk.  Two launches: a chunk kernel and, for multi-chunk rows,
+ *   a combine kernel.
  */
 int archer_decode_scores(int batch, int resp_len, int vocab, int dtype, const void* logits,
                          int64_t row_stride, const uint8_t* mask_state, const int32_t* cur_tokens,
@@ -143,9 +145,10 @@ size_t archer_decode_scores_workspace_size(int rows, int vocab);
  *   The first call on a device looks up the array's device address (this may
  *   load the library's device code on that device); make that first call
  *   before any stream capture.
- *   Every call shares the one array per device and clears its counters on
- *   `stream` before launching: calls that can overlap on the GPU (other
- *   streams, other host threads) race and must be serialised by the caller.
+ *   Every call shares the one array per device (which keeps the last call's
+ *   partials; nothing in it needs clearing): calls that can overlap on the GPU
+ *   (other streams, other host threads) race and must be serialised by the
+ *   caller.
  *   Calls no cudaMalloc / cudaFree.
  */
 #define ARCHER_NOALLOC_SCRATCH_BYTES (4u << 20)

@@ -11,9 +11,10 @@
 //     with packed bf16x2 max/min, 1.5 ops per element), CTA-reduced;
 //   * pass B: sum of 2^((z - m) log2 e) with the CTA max m -- exactly one ex2
 //     per element; the lowest index of m is found by the threads holding it;
-//   * chunk partials (m, sum, top-2 value, index) go to the workspace; the
-//     last CTA of a row (ticket counter) merges them and writes the outputs
-//     and re-zeroes the counter.  A row of one chunk skips the workspace.
+//   * chunk partials (m, sum, top-2 value, index) go to the workspace and the
+//     CTA exits at once -- no CTA waits on another, so HBM reads stay in
+//     flight; a combine kernel (one warp per row) then merges each row's
+//     partials and writes the outputs.  A row of one chunk skips both.
 
 #include <cfloat>
 #include <cmath>
@@ -151,8 +152,7 @@ __global__ void __launch_bounds__(kThreads)
 decode_scores_kernel(const T* __restrict__ logits, int64_t row_stride, int vocab, int chunks,
                      const uint8_t* __restrict__ mask_state, const int32_t* __restrict__ cur_tokens,
                      float* __restrict__ max_prob, int32_t* __restrict__ top1, float* __restrict__ margin,
-                     float* __restrict__ cur_prob, int* __restrict__ counters, Partial* __restrict__ parts,
-                     int aligned) {
+                     float* __restrict__ cur_prob, Partial* __restrict__ parts, int aligned) {
   constexpr int E = Vec<T>::kElems;              // elements per 16-byte word
   constexpr int dtype = sizeof(T) == 2 ? ARCHER_DTYPE_BF16 : ARCHER_DTYPE_F32;
   __shared__ Smem sm;
@@ -249,46 +249,50 @@ decode_scores_kernel(const T* __restrict__ logits, int64_t row_stride, int vocab
     return;
   }
 
-  // ---- publish the chunk partial; the last CTA of the row merges
+  // ---- publish the chunk partial and leave: no CTA waits on another one
   if (threadIdx.x == 0) {
     Partial pt;
     pt.m = m_blk; pt.s = s; pt.t2 = t2_blk; pt.idx = idx;
     parts[static_cast<size_t>(row) * chunks + chunk] = pt;
-    __threadfence();
-    const int ticket = atomicAdd(&counters[row], 1);
-    sm.last = (ticket == chunks - 1);
   }
-  __syncthreads();
-  if (!sm.last) return;
-  __threadfence();
-  if (threadIdx.x < 32) {
-    // warp 0 merges the chunk partials of this row
-    float M = -INFINITY, T2 = -INFINITY;
-    const volatile Partial* vp = parts + static_cast<size_t>(row) * chunks;
-    for (int c = threadIdx.x; c < chunks; c += 32) merge_top2(M, T2, vp[c].m, vp[c].t2);
+}
+
+// One warp per row merges the row's chunk partials (launched after the chunk
+// kernel on the same stream).
+template <typename T>
+__global__ void __launch_bounds__(256)
+decode_scores_combine_kernel(const T* __restrict__ logits, int64_t row_stride, int vocab, int chunks, int rows,
+                             const uint8_t* __restrict__ mask_state, const int32_t* __restrict__ cur_tokens,
+                             float* __restrict__ max_prob, int32_t* __restrict__ top1, float* __restrict__ margin,
+                             float* __restrict__ cur_prob, const Partial* __restrict__ parts) {
+  constexpr int dtype = sizeof(T) == 2 ? ARCHER_DTYPE_BF16 : ARCHER_DTYPE_F32;
+  const int row = blockIdx.x * 8 + (threadIdx.x >> 5);
+  const int l = threadIdx.x & 31;
+  if (row >= rows) return;
+  const Partial* vp = parts + static_cast<size_t>(row) * chunks;
+  float M = -INFINITY, T2 = -INFINITY;
+  for (int c = l; c < chunks; c += 32) merge_top2(M, T2, vp[c].m, vp[c].t2);
 #pragma unroll
-    for (int o = 16; o > 0; o >>= 1) {
-      const float b1 = __shfl_xor_sync(0xffffffffu, M, o);
-      const float b2 = __shfl_xor_sync(0xffffffffu, T2, o);
-      merge_top2(M, T2, b1, b2);
-    }
-    float S = 0.f;
-    int I = INT_MAX;
-    for (int c = threadIdx.x; c < chunks; c += 32) {
-      const float mc = vp[c].m;
-      S += vp[c].s * ex2_approx((mc - M) * kLog2e);
-      if (mc == M) I = min(I, (int)vp[c].idx);
-    }
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) {
-      S += __shfl_xor_sync(0xffffffffu, S, o);
-      I = min(I, __shfl_xor_sync(0xffffffffu, I, o));
-    }
-    if (threadIdx.x == 0) {
-      write_row(row, M, S, T2, I, zrow, dtype, vocab, mask_state, cur_tokens, max_prob, top1, margin, cur_prob);
-      counters[row] = 0;   // leave the workspace zero-filled for the next call
-    }
+  for (int o = 16; o > 0; o >>= 1) {
+    const float b1 = __shfl_xor_sync(0xffffffffu, M, o);
+    const float b2 = __shfl_xor_sync(0xffffffffu, T2, o);
+    merge_top2(M, T2, b1, b2);
   }
+  float S = 0.f;
+  int I = INT_MAX;
+  for (int c = l; c < chunks; c += 32) {
+    const float mc = vp[c].m;
+    if (mc != -INFINITY) S += vp[c].s * ex2_approx((mc - M) * kLog2e);
+    if (mc == M) I = min(I, vp[c].idx);
+  }
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) {
+    S += __shfl_xor_sync(0xffffffffu, S, o);
+    I = min(I, __shfl_xor_sync(0xffffffffu, I, o));
+  }
+  if (l == 0)
+    write_row(row, M, S, T2, I, logits + row * row_stride, dtype, vocab, mask_state, cur_tokens, max_prob, top1,
+              margin, cur_prob);
 }
 
 int chunks_for(int vocab, int dtype) {
@@ -302,8 +306,7 @@ size_t decode_scores_ws_bytes(int rows, int vocab) {
   // Sized for fp32 logits, which need twice the chunks of bf16 for one vocabulary.
   const int chunks = chunks_for(vocab, ARCHER_DTYPE_F32);
   if (chunks <= 1 || rows <= 0) return 0;
-  const size_t counters = ((static_cast<size_t>(rows) * sizeof(int) + 255) / 256) * 256;
-  return counters + static_cast<size_t>(rows) * chunks * sizeof(Partial);
+  return static_cast<size_t>(rows) * chunks * sizeof(Partial);
 }
 
 int decode_scores_launch(int rows, int vocab, int dtype, const void* logits, int64_t row_stride,
@@ -311,17 +314,14 @@ int decode_scores_launch(int rows, int vocab, int dtype, const void* logits, int
                          float* margin, float* cur_prob, void* workspace, size_t ws_bytes, cudaStream_t stream) {
   if (rows == 0) return ARCHER_OK;
   const int chunks = chunks_for(vocab, dtype);
-  int* counters = nullptr;
   Partial* parts = nullptr;
   if (chunks > 1) {
     const size_t need = decode_scores_ws_bytes(rows, vocab);
     if (workspace == nullptr || ws_bytes < need) {
-      set_error("decode_scores needs a zero-filled workspace of %zu bytes (got %zu)", need, ws_bytes);
+      set_error("decode_scores needs a workspace of %zu bytes (got %zu)", need, ws_bytes);
       return ARCHER_ERR_ARG;
     }
-    counters = static_cast<int*>(workspace);
-    parts = reinterpret_cast<Partial*>(static_cast<char*>(workspace) +
-                                       ((static_cast<size_t>(rows) * sizeof(int) + 255) / 256) * 256);
+    parts = static_cast<Partial*>(workspace);
   }
   const int esize = dtype == ARCHER_DTYPE_BF16 ? 2 : 4;
   const int aligned = (reinterpret_cast<uintptr_t>(logits) % 16 == 0) && ((row_stride * esize) % 16 == 0);
@@ -330,14 +330,23 @@ int decode_scores_launch(int rows, int vocab, int dtype, const void* logits, int
     set_error("decode_scores grid too large");
     return ARCHER_ERR_UNSUPPORTED;
   }
+  const unsigned combine_grid = static_cast<unsigned>((rows + 7) / 8);
   if (dtype == ARCHER_DTYPE_BF16) {
     decode_scores_kernel<__nv_bfloat16><<<(unsigned)grid, kThreads, 0, stream>>>(
         static_cast<const __nv_bfloat16*>(logits), row_stride, vocab, chunks, mask_state, cur_tokens, max_prob, top1,
-        margin, cur_prob, counters, parts, aligned);
+        margin, cur_prob, parts, aligned);
+    if (chunks > 1)
+      decode_scores_combine_kernel<__nv_bfloat16><<<combine_grid, 256, 0, stream>>>(
+          static_cast<const __nv_bfloat16*>(logits), row_stride, vocab, chunks, rows, mask_state, cur_tokens,
+          max_prob, top1, margin, cur_prob, parts);
   } else {
     decode_scores_kernel<float><<<(unsigned)grid, kThreads, 0, stream>>>(
         static_cast<const float*>(logits), row_stride, vocab, chunks, mask_state, cur_tokens, max_prob, top1, margin,
-        cur_prob, counters, parts, aligned);
+        cur_prob, parts, aligned);
+    if (chunks > 1)
+      decode_scores_combine_kernel<float><<<combine_grid, 256, 0, stream>>>(
+          static_cast<const float*>(logits), row_stride, vocab, chunks, rows, mask_state, cur_tokens, max_prob, top1,
+          margin, cur_prob, parts);
   }
   return cuda_status(cudaGetLastError(), "decode_scores launch");
 }
@@ -351,7 +360,7 @@ int decode_scores_launch(int rows, int vocab, int dtype, const void* logits, int
 // inside another framework's memory pool (where a raw cudaMalloc bypasses its
 // accounting), latency-critical loops that must not pay cudaMalloc's implicit
 // device synchronisation, and thin foreign-function bindings with no allocator
-// at hand.  For them the chunk partials and ticket counters live in this
+// at hand.  For them the chunk partials live in this
 // file-scope array, created when the library is loaded on a device and held
 // by every GPU that loads the library until the process exits.
 // ---------------------------------------------------------------------------
@@ -414,14 +423,8 @@ extern "C" int archer_decode_scores_noalloc(int batch, int resp_len, int vocab, 
   void* scratch = nullptr;
   int st = scratch_address(&scratch);
   if (st) return st;
-  const cudaStream_t s = static_cast<cudaStream_t>(stream);
-  if (need > 0) {
-    // The ticket counters must start at zero; a call normally leaves them so,
-    // but clear them in case an earlier call on this device did not finish.
-    const size_t counter_bytes = ((static_cast<size_t>(rows) * sizeof(int) + 255) / 256) * 256;
-    cudaError_t e = cudaMemsetAsync(scratch, 0, counter_bytes, s);
-    if (e != cudaSuccess) return cuda_status(e, "clearing the scoring scratch counters");
-  }
+  // Every chunk partial is written before the combine kernel reads it, so the
+  // scratch needs no clearing between calls.
   return archer_decode_scores(batch, resp_len, vocab, dtype, logits, row_stride, mask_state, cur_tokens, max_prob,
                               top1, margin, cur_prob, scratch, kNoAllocScratchBytes, stream);
 }
