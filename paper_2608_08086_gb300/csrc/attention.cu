@@ -18,8 +18,9 @@
 //              is written over S's own TMEM columns and handed to the MMA warp
 //              at once, so P V of the first half overlaps the second half's
 //              exponentials.
-//   warp 8     TMA producer: Q_A, Q_B once, then K tiles (3-stage ring) and V
-//              tiles (2-stage ring) of 128 keys.
+//   warp 8     TMA producer: Q_A, Q_B once, then K_0, V_0, K_1, V_1, ... tiles
+//              of 128 keys through one 5-slot ring (about two tiles of
+//              lookahead for both K and V).
 //   warp 9     MMA issuer (one thread), per K/V tile j:
 //                PV_A(j) in two halves, QK_A(j+1), PV_B(j) in two halves, QK_B(j+1)
 //              so the tensor pipe works on one tile while the other tile's
@@ -70,14 +71,12 @@ template <int D>
 struct Layout {
   static constexpr int kChunks = D / 64;                    // 128-byte column chunks
   static constexpr uint32_t kTile = kChunks * kChunkBytes;  // one 128-row tile of D bf16
-  static constexpr int kKS = 3, kVS = 2;                    // K / V ring stages
+  static constexpr int kSlots = 5;                          // K/V ring: item 2j = K_j, 2j+1 = V_j
   static constexpr uint32_t kOffQ = 0;                      // Q_A, Q_B
-  static constexpr uint32_t kOffK = kOffQ + 2 * kTile;
-  static constexpr uint32_t kOffV = kOffK + kKS * kTile;
-  static constexpr uint32_t kOffBar = kOffV + kVS * kTile;
-  // q_full, k_full[KS], k_empty[KS], v_full[VS], v_empty[VS],
-  // s_full[2], p_half0[2], p_half1[2], pv_half0_done[2]
-  static constexpr int kBars = 1 + 2 * kKS + 2 * kVS + 8;
+  static constexpr uint32_t kOffKV = kOffQ + 2 * kTile;
+  static constexpr uint32_t kOffBar = kOffKV + kSlots * kTile;
+  // q_full, full[slots], empty[slots], s_full[2], p_half0[2], p_half1[2], pv_half0_done[2]
+  static constexpr int kBars = 1 + 2 * kSlots + 8;
   static constexpr uint32_t kOffHolder = kOffBar + 8 * kBars;
   static constexpr uint32_t kOffAbort = kOffHolder + 4;
   static constexpr uint32_t kUsed = kOffAbort + 4;
@@ -177,15 +176,12 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
   const uint32_t base = (raw + 1023u) & ~1023u;
   uint8_t* gbase = smem_raw + (base - raw);
   const uint32_t sQ = base + L::kOffQ;
-  const uint32_t sK = base + L::kOffK;
-  const uint32_t sV = base + L::kOffV;
+  const uint32_t sKV = base + L::kOffKV;
   const uint32_t bars = base + L::kOffBar;
   const uint32_t bar_q_full = bars;
-  const uint32_t bar_k_full = bars + 8;                         // + 8 * stage
-  const uint32_t bar_k_empty = bar_k_full + 8 * L::kKS;
-  const uint32_t bar_v_full = bar_k_empty + 8 * L::kKS;
-  const uint32_t bar_v_empty = bar_v_full + 8 * L::kVS;
-  const uint32_t bar_s_full = bar_v_empty + 8 * L::kVS;         // + 8 * tile (A = 0, B = 1)
+  const uint32_t bar_full = bars + 8;                           // + 8 * slot
+  const uint32_t bar_empty = bar_full + 8 * L::kSlots;          // + 8 * slot
+  const uint32_t bar_s_full = bar_empty + 8 * L::kSlots;        // + 8 * tile (A = 0, B = 1)
   const uint32_t bar_p_h0 = bar_s_full + 16;                    // + 8 * tile: first half of P written
   const uint32_t bar_p_h1 = bar_p_h0 + 16;                      // + 8 * tile: second half of P written
   const uint32_t bar_pv_h0 = bar_p_h1 + 16;                     // + 8 * tile: P V of the first half done
@@ -195,13 +191,9 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
   const int warp = threadIdx.x >> 5;
   if (threadIdx.x == 0) {
     mbar_init(bar_q_full, 1);
-    for (int s = 0; s < L::kKS; ++s) {
-      mbar_init(bar_k_full + 8 * s, 1);
-      mbar_init(bar_k_empty + 8 * s, 1);
-    }
-    for (int s = 0; s < L::kVS; ++s) {
-      mbar_init(bar_v_full + 8 * s, 1);
-      mbar_init(bar_v_empty + 8 * s, 1);
+    for (int s = 0; s < L::kSlots; ++s) {
+      mbar_init(bar_full + 8 * s, 1);
+      mbar_init(bar_empty + 8 * s, 1);
     }
     for (int i = 0; i < 2; ++i) {
       mbar_init(bar_s_full + 8 * i, 1);
@@ -231,21 +223,17 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
       for (int t = 0; t < (has_b ? 2 : 1); ++t)
         for (int c = 0; c < L::kChunks; ++c)
           tma_load_4d(sQ + t * L::kTile + c * kChunkBytes, &tmQ, bar_q_full, c * 64, h, q0 + t * kBM, b);
-      for (int j = 0; j < T; ++j) {
+      for (int item = 0; item < 2 * T; ++item) {
+        const int j = item >> 1;
+        const bool is_v = item & 1;
         const bool in_prompt = j < n_p;
         const int row = in_prompt ? j * kBN : (j - n_p) * kBN;
-        const int ks = j % L::kKS, kuse = j / L::kKS;
-        if (kuse > 0 && !mbar_wait(bar_k_empty + 8 * ks, (kuse - 1) & 1, abort, p.err, p.wait_limit)) break;
-        mbar_arrive_expect_tx(bar_k_full + 8 * ks, L::kTile);
-        const CUtensorMap* mk = in_prompt ? mKp : &tmKg;
+        const int slot = item % L::kSlots, use = item / L::kSlots;
+        if (use > 0 && !mbar_wait(bar_empty + 8 * slot, (use - 1) & 1, abort, p.err, p.wait_limit)) break;
+        mbar_arrive_expect_tx(bar_full + 8 * slot, L::kTile);
+        const CUtensorMap* map = in_prompt ? (is_v ? mVp : mKp) : (is_v ? &tmVg : &tmKg);
         for (int c = 0; c < L::kChunks; ++c)
-          tma_load_4d(sK + ks * L::kTile + c * kChunkBytes, mk, bar_k_full + 8 * ks, c * 64, kvh, row, b);
-        const int vs = j % L::kVS, vuse = j / L::kVS;
-        if (vuse > 0 && !mbar_wait(bar_v_empty + 8 * vs, (vuse - 1) & 1, abort, p.err, p.wait_limit)) break;
-        mbar_arrive_expect_tx(bar_v_full + 8 * vs, L::kTile);
-        const CUtensorMap* mv = in_prompt ? mVp : &tmVg;
-        for (int c = 0; c < L::kChunks; ++c)
-          tma_load_4d(sV + vs * L::kTile + c * kChunkBytes, mv, bar_v_full + 8 * vs, c * 64, kvh, row, b);
+          tma_load_4d(sKV + slot * L::kTile + c * kChunkBytes, map, bar_full + 8 * slot, c * 64, kvh, row, b);
       }
     }
     __syncwarp();
@@ -273,43 +261,47 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
                   idesc_pv, (acc || kk > 0) ? 1u : 0u);
         }
       };
+      // K_j is ring item 2j, V_j item 2j + 1.
+      auto slot_of = [](int item) { return item % L::kSlots; };
+      auto phase_of = [](int item) { return static_cast<uint32_t>(item / L::kSlots) & 1u; };
       bool ok = mbar_wait(bar_q_full, 0, abort, p.err, p.wait_limit) &&
-                mbar_wait(bar_k_full, 0, abort, p.err, p.wait_limit);
+                mbar_wait(bar_full + 8 * slot_of(0), phase_of(0), abort, p.err, p.wait_limit);
       if (ok) {
         tc_fence_after();
         for (int t = 0; t < n_tiles; ++t) {
-          issue_qk(t, sK);
+          issue_qk(t, sKV + slot_of(0) * L::kTile);
           umma_commit(bar_s_full + 8 * t);
         }
-        umma_commit(bar_k_empty);
+        umma_commit(bar_empty + 8 * slot_of(0));
       }
       for (int j = 0; ok && j < T; ++j) {
-        const int vs = j % L::kVS;
         const bool more = j + 1 < T;
-        const int ks = (j + 1) % L::kKS;
-        if (!mbar_wait(bar_v_full + 8 * vs, (j / L::kVS) & 1, abort, p.err, p.wait_limit)) break;
+        const int v_item = 2 * j + 1, k_item = 2 * j + 2;
+        const uint32_t v_tile = sKV + slot_of(v_item) * L::kTile;
+        const uint32_t k_tile = sKV + slot_of(k_item) * L::kTile;
+        if (!mbar_wait(bar_full + 8 * slot_of(v_item), phase_of(v_item), abort, p.err, p.wait_limit)) break;
         for (int t = 0; t < n_tiles; ++t) {
           if (!mbar_wait(bar_p_h0 + 8 * t, j & 1, abort, p.err, p.wait_limit)) { ok = false; break; }
           if (p.debug_skip_last_pv && !more) { ok = false; break; }   // the softmax's final wait must expire
           tc_fence_after();
-          issue_pv(t, 0, sV + vs * L::kTile, j > 0);
+          issue_pv(t, 0, v_tile, j > 0);
           umma_commit(bar_pv_h0 + 8 * t);
           if (!mbar_wait(bar_p_h1 + 8 * t, j & 1, abort, p.err, p.wait_limit)) { ok = false; break; }
           tc_fence_after();
-          issue_pv(t, 1, sV + vs * L::kTile, true);
+          issue_pv(t, 1, v_tile, true);
           if (more) {
-            if (t == 0 && !mbar_wait(bar_k_full + 8 * ks, ((j + 1) / L::kKS) & 1, abort, p.err, p.wait_limit)) {
+            if (t == 0 && !mbar_wait(bar_full + 8 * slot_of(k_item), phase_of(k_item), abort, p.err, p.wait_limit)) {
               ok = false;
               break;
             }
             tc_fence_after();
-            issue_qk(t, sK + ks * L::kTile);
+            issue_qk(t, k_tile);
           }
           umma_commit(bar_s_full + 8 * t);   // S_t(j+1) ready -- or, after the last tile, O_t final
         }
         if (!ok) break;
-        umma_commit(bar_v_empty + 8 * vs);
-        if (more) umma_commit(bar_k_empty + 8 * ks);
+        umma_commit(bar_empty + 8 * slot_of(v_item));
+        if (more) umma_commit(bar_empty + 8 * slot_of(k_item));
       }
     }
     __syncwarp();
