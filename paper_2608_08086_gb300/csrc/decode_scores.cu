@@ -257,6 +257,141 @@ decode_scores_kernel(const T* __restrict__ logits, int64_t row_stride, int vocab
   }
 }
 
+// Aligned-row variant: one TMA bulk copy stages the CTA's chunk in shared
+// memory, so no registers are held while the chunk is in flight and six CTAs
+// per SM keep about 192 KB of reads outstanding.  Same partition, partials
+// and arithmetic as decode_scores_kernel.
+constexpr uint32_t kBulkBytes = kWordsPerChunk * 16;   // 32 KB
+
+__device__ __forceinline__ void bulk_load(uint32_t dst, const void* src, uint32_t bytes, uint32_t bar) {
+  asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(dst),
+               "l"(reinterpret_cast<uint64_t>(src)), "r"(bytes), "r"(bar)
+               : "memory");
+}
+
+template <typename T>
+__global__ void __launch_bounds__(kThreads, 6)
+decode_scores_bulk_kernel(const T* __restrict__ logits, int64_t row_stride, int vocab, int chunks,
+                          const uint8_t* __restrict__ mask_state, const int32_t* __restrict__ cur_tokens,
+                          float* __restrict__ max_prob, int32_t* __restrict__ top1, float* __restrict__ margin,
+                          float* __restrict__ cur_prob, Partial* __restrict__ parts, int* __restrict__ err) {
+  constexpr int E = Vec<T>::kElems;
+  constexpr int dtype = sizeof(T) == 2 ? ARCHER_DTYPE_BF16 : ARCHER_DTYPE_F32;
+  constexpr int kChunkElems = kWordsPerChunk * E;
+  extern __shared__ __align__(128) uint4 stage[];
+  __shared__ Smem sm;
+  __shared__ __align__(8) uint64_t full_bar;
+  __shared__ int abort_flag;
+  const int row = blockIdx.x / chunks;
+  const int chunk = blockIdx.x - row * chunks;
+  const T* zrow = logits + row * row_stride;
+  const int64_t e0c = static_cast<int64_t>(chunk) * kChunkElems;
+  const int n_el = static_cast<int>(min(static_cast<int64_t>(kChunkElems), static_cast<int64_t>(vocab) - e0c));
+  const uint32_t bytes = (static_cast<uint32_t>(n_el) * sizeof(T)) & ~15u;
+  const int bulk_words = static_cast<int>(bytes / 16);
+  const uint32_t bar = smem_u32(&full_bar);
+  if (threadIdx.x == 0) {
+    abort_flag = 0;
+    mbar_init(bar, 1);
+    mbar_fence_init();
+    if (bytes > 0) {
+      mbar_arrive_expect_tx(bar, bytes);
+      bulk_load(smem_u32(stage), zrow + e0c, bytes, bar);
+    } else {
+      mbar_arrive(bar);
+    }
+  }
+  __syncthreads();
+  // An expired wait is reported through the error word; the CTA then reads
+  // stale shared memory (in bounds) rather than leaving early.
+  mbar_wait(bar, 0, &abort_flag, err);
+
+  auto word = [&](int u) -> uint4 {
+    const int wi = u * kThreads + threadIdx.x;
+    if (wi < bulk_words) return stage[wi];
+    float v[E];
+#pragma unroll
+    for (int e = 0; e < E; ++e) {
+      const int el = wi * E + e;
+      v[e] = (el < n_el) ? load_logit(zrow, dtype, static_cast<int>(e0c + el)) : -INFINITY;
+    }
+    if constexpr (E == 8) {
+      return make_uint4(pack_bf16x2(v[0], v[1]), pack_bf16x2(v[2], v[3]), pack_bf16x2(v[4], v[5]),
+                        pack_bf16x2(v[6], v[7]));
+    } else {
+      return make_uint4(__float_as_uint(v[0]), __float_as_uint(v[1]), __float_as_uint(v[2]), __float_as_uint(v[3]));
+    }
+  };
+
+  // pass A: top-2 values
+  float t1 = -INFINITY, t2 = -INFINITY;
+  if constexpr (E == 8) {
+    __nv_bfloat162 M1 = __floats2bfloat162_rn(-INFINITY, -INFINITY);
+    __nv_bfloat162 M2 = M1;
+#pragma unroll
+    for (int u = 0; u < kUnroll; ++u) {
+      const uint4 wv = word(u);
+      const uint32_t q[4] = {wv.x, wv.y, wv.z, wv.w};
+#pragma unroll
+      for (int i = 0; i < 4; ++i) {
+        const __nv_bfloat162 x = *reinterpret_cast<const __nv_bfloat162*>(&q[i]);
+        M2 = __hmax2(M2, __hmin2(M1, x));
+        M1 = __hmax2(M1, x);
+      }
+    }
+    const float a = __low2float(M1), c = __high2float(M1);
+    t1 = fmaxf(a, c);
+    t2 = fmaxf(fminf(a, c), fmaxf(__low2float(M2), __high2float(M2)));
+  } else {
+#pragma unroll
+    for (int u = 0; u < kUnroll; ++u) {
+      float v[4];
+      unpack(word(u), v, (float*)nullptr);
+#pragma unroll
+      for (int e = 0; e < 4; ++e) {
+        t2 = fmaxf(t2, fminf(t1, v[e]));
+        t1 = fmaxf(t1, v[e]);
+      }
+    }
+  }
+  const float my_t1 = t1;
+  float m_blk = t1, t2_blk = t2;
+  block_top2(m_blk, t2_blk, sm);
+
+  // pass B: one ex2 per logit against the chunk max; lowest index of the max
+  const float neg_m = (m_blk == -INFINITY) ? 0.f : -m_blk * kLog2e;
+  float sum = 0.f;
+#pragma unroll
+  for (int u = 0; u < kUnroll; ++u) {
+    float v[E];
+    unpack(word(u), v, (T*)nullptr);
+#pragma unroll
+    for (int e = 0; e < E; ++e) sum += ex2_approx(fmaf(v[e], kLog2e, neg_m));
+  }
+  int idx = INT_MAX;
+  if (my_t1 == m_blk) {
+    for (int u = 0; u < kUnroll && idx == INT_MAX; ++u) {
+      float v[E];
+      unpack(word(u), v, (T*)nullptr);
+      const int64_t el0 = e0c + static_cast<int64_t>(u * kThreads + threadIdx.x) * E;
+#pragma unroll
+      for (int e = E - 1; e >= 0; --e)
+        if (v[e] == m_blk) idx = static_cast<int>(el0 + e);
+    }
+  }
+  block_sum_minidx(sum, idx, sm);
+  if (threadIdx.x == 0) {
+    if (chunks == 1) {
+      write_row(row, m_blk, sum, t2_blk, idx, zrow, dtype, vocab, mask_state, cur_tokens, max_prob, top1, margin,
+                cur_prob);
+    } else {
+      Partial pt;
+      pt.m = m_blk; pt.s = sum; pt.t2 = t2_blk; pt.idx = idx;
+      parts[static_cast<size_t>(row) * chunks + chunk] = pt;
+    }
+  }
+}
+
 // One warp per row merges the row's chunk partials (launched after the chunk
 // kernel on the same stream).
 template <typename T>
@@ -331,6 +466,27 @@ int decode_scores_launch(int rows, int vocab, int dtype, const void* logits, int
     return ARCHER_ERR_UNSUPPORTED;
   }
   const unsigned combine_grid = static_cast<unsigned>((rows + 7) / 8);
+  if (aligned) {
+    if (dtype == ARCHER_DTYPE_BF16)
+      decode_scores_bulk_kernel<__nv_bfloat16><<<(unsigned)grid, kThreads, kBulkBytes, stream>>>(
+          static_cast<const __nv_bfloat16*>(logits), row_stride, vocab, chunks, mask_state, cur_tokens, max_prob,
+          top1, margin, cur_prob, parts, device_error_word());
+    else
+      decode_scores_bulk_kernel<float><<<(unsigned)grid, kThreads, kBulkBytes, stream>>>(
+          static_cast<const float*>(logits), row_stride, vocab, chunks, mask_state, cur_tokens, max_prob, top1,
+          margin, cur_prob, parts, device_error_word());
+    if (chunks > 1) {
+      if (dtype == ARCHER_DTYPE_BF16)
+        decode_scores_combine_kernel<__nv_bfloat16><<<combine_grid, 256, 0, stream>>>(
+            static_cast<const __nv_bfloat16*>(logits), row_stride, vocab, chunks, rows, mask_state, cur_tokens,
+            max_prob, top1, margin, cur_prob, parts);
+      else
+        decode_scores_combine_kernel<float><<<combine_grid, 256, 0, stream>>>(
+            static_cast<const float*>(logits), row_stride, vocab, chunks, rows, mask_state, cur_tokens, max_prob,
+            top1, margin, cur_prob, parts);
+    }
+    return cuda_status(cudaGetLastError(), "decode_scores launch");
+  }
   if (dtype == ARCHER_DTYPE_BF16) {
     decode_scores_kernel<__nv_bfloat16><<<(unsigned)grid, kThreads, 0, stream>>>(
         static_cast<const __nv_bfloat16*>(logits), row_stride, vocab, chunks, mask_state, cur_tokens, max_prob, top1,
