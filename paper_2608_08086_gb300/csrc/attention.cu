@@ -9,19 +9,19 @@
 // formed in memory.  GQA: query head h reads KV head h / (Hq / Hkv).
 //
 // One CTA = two 128-row query tiles (A and B) of one (b, h) sharing every K/V
-// tile; 10 warps:
-//   warps 0-3  softmax of tile A, warps 4-7 softmax of tile B: thread t of a
-//              warpgroup owns query row t (TMEM lane t).  S is read in two
-//              64-column halves; exponentials use the running max in use and
-//              the max is raised lazily (only when a half's max exceeds it by
-//              more than 2^8), rescaling l and O.  Each half of P (bf16 pairs)
-//              is written over S's own TMEM columns and handed to the MMA warp
-//              at once, so P V of the first half overlaps the second half's
-//              exponentials.
-//   warp 8     TMA producer: Q_A, Q_B once, then K_0, V_0, K_1, V_1, ... tiles
-//              of 128 keys through one 5-slot ring (about two tiles of
-//              lookahead for both K and V).
-//   warp 9     MMA issuer (one thread), per K/V tile j:
+// tile; 18 warps:
+//   warps 0-15 softmax: four warpgroups, (tile A, keys 0-63), (A, 64-127),
+//              (B, 0-63), (B, 64-127).  Thread t of a warpgroup owns query row
+//              t (TMEM lane t) for its 64 key columns.  The two groups of a
+//              tile exchange their row maxima through shared memory (a named
+//              barrier per tile); exponentials use the running max in use,
+//              raised lazily (only when the tile max exceeds it by more than
+//              2^8, rescaling l and each group's half of O).  Each group writes
+//              its half of P (bf16 pairs) over the first 32 of its own 64 S
+//              columns and hands it to the MMA warp at once.
+//   warp 16    TMA producer: Q_A, Q_B once, then K_0, V_0, K_1, V_1, ... tiles
+//              of 128 keys through one 4-slot ring.
+//   warp 17    MMA issuer (one thread), per K/V tile j:
 //                PV_A(j) in two halves, QK_A(j+1), PV_B(j) in two halves, QK_B(j+1)
 //              so the tensor pipe works on one tile while the other tile's
 //              softmax runs.  tcgen05.mma executes in issue order, so QK_X(j+1)
@@ -47,8 +47,8 @@ namespace {
 
 constexpr int kBM = 128;          // query rows per tile (tcgen05 M)
 constexpr int kBN = 128;          // keys per KV tile (N of Q K^T, K of P V)
-constexpr int kThreads = 320;     // 2 softmax warpgroups + producer warp + MMA warp
-constexpr int kWarpProducer = 8, kWarpMma = 9;
+constexpr int kThreads = 576;     // 4 softmax warpgroups + producer warp + MMA warp
+constexpr int kWarpProducer = 16, kWarpMma = 17;
 constexpr uint32_t kTmemCols = 512;
 // TMEM columns of tile t's S (P is written over its first 64 columns) and O.
 __host__ __device__ constexpr uint32_t col_s(int t) { return 128u * static_cast<uint32_t>(t); }
@@ -71,13 +71,14 @@ template <int D>
 struct Layout {
   static constexpr int kChunks = D / 64;                    // 128-byte column chunks
   static constexpr uint32_t kTile = kChunks * kChunkBytes;  // one 128-row tile of D bf16
-  static constexpr int kSlots = 5;                          // K/V ring: item 2j = K_j, 2j+1 = V_j
+  static constexpr int kSlots = 4;                          // K/V ring: item 2j = K_j, 2j+1 = V_j
   static constexpr uint32_t kOffQ = 0;                      // Q_A, Q_B
   static constexpr uint32_t kOffKV = kOffQ + 2 * kTile;
   static constexpr uint32_t kOffBar = kOffKV + kSlots * kTile;
-  // q_full, full[slots], empty[slots], s_full[2], p_half0[2], p_half1[2], pv_half0_done[2]
-  static constexpr int kBars = 1 + 2 * kSlots + 8;
-  static constexpr uint32_t kOffHolder = kOffBar + 8 * kBars;
+  // q_full, full[slots], empty[slots], s_full[2], p_half0[2], p_half1[2]
+  static constexpr int kBars = 1 + 2 * kSlots + 6;
+  static constexpr uint32_t kOffXch = kOffBar + 8 * kBars;  // [tile parity][tile][half][row] floats
+  static constexpr uint32_t kOffHolder = kOffXch + 2 * 2 * 2 * 128 * 4;
   static constexpr uint32_t kOffAbort = kOffHolder + 4;
   static constexpr uint32_t kUsed = kOffAbort + 4;
   // + 1 KB to align the base to 1024 B; at least 120 KB so that one CTA
@@ -105,17 +106,15 @@ __device__ __forceinline__ bool warp_wait(uint32_t bar, uint32_t parity, volatil
   }
 }
 
+// Named barrier for the 256 softmax threads of tile t (ids 1 and 2; 0 is __syncthreads).
+__device__ __forceinline__ void tile_bar(int t) {
+  asm volatile("bar.sync %0, 256;" ::"r"(1 + t) : "memory");
+}
+
 __device__ __forceinline__ float max3f(float a, float b, float c) {
   float d;
   asm("max.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));
   return d;
-}
-
-__device__ __forceinline__ float max64(const float (&x)[64]) {
-  float m[4] = {x[0], x[1], x[2], x[3]};
-#pragma unroll
-  for (int c = 4; c < 64; c += 2) m[(c >> 1) & 3] = max3f(m[(c >> 1) & 3], x[c], x[c + 1]);
-  return max3f(m[0], m[1], fmaxf(m[2], m[3]));
 }
 
 // Packed fp32 pairs (two lanes per instruction).
@@ -138,15 +137,22 @@ __device__ __forceinline__ float2 fadd2(float2 a, float2 b) {
   return d;
 }
 
-// Loads 64 score columns [c0, c0 + 64) of this lane and masks keys >= valid.
-__device__ __forceinline__ void load_scores(uint32_t taddr, int c0, int valid, float (&x)[64]) {
-  uint32_t r[64];
-  tmem_ld_64(taddr, r);
+__device__ __forceinline__ float max32(const float (&x)[32]) {
+  float m[4] = {x[0], x[1], x[2], x[3]};
 #pragma unroll
-  for (int c = 0; c < 64; ++c) x[c] = __uint_as_float(r[c]);
-  if (valid < c0 + 64) {            // only the last tile of a segment is ragged
+  for (int c = 4; c < 32; c += 2) m[(c >> 1) & 3] = max3f(m[(c >> 1) & 3], x[c], x[c + 1]);
+  return max3f(m[0], m[1], fmaxf(m[2], m[3]));
+}
+
+// Loads 32 score columns [c0, c0 + 32) of this lane and masks keys >= valid.
+__device__ __forceinline__ void load_scores32(uint32_t taddr, int c0, int valid, float (&x)[32]) {
+  uint32_t r[32];
+  tmem_ld_32(taddr, r);
 #pragma unroll
-    for (int c = 0; c < 64; ++c)
+  for (int c = 0; c < 32; ++c) x[c] = __uint_as_float(r[c]);
+  if (valid < c0 + 32) {            // only the last tile of a segment is ragged
+#pragma unroll
+    for (int c = 0; c < 32; ++c)
       if (c0 + c >= valid) x[c] = -INFINITY;
   }
 }
@@ -184,7 +190,7 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
   const uint32_t bar_s_full = bar_empty + 8 * L::kSlots;        // + 8 * tile (A = 0, B = 1)
   const uint32_t bar_p_h0 = bar_s_full + 16;                    // + 8 * tile: first half of P written
   const uint32_t bar_p_h1 = bar_p_h0 + 16;                      // + 8 * tile: second half of P written
-  const uint32_t bar_pv_h0 = bar_p_h1 + 16;                     // + 8 * tile: P V of the first half done
+  float* xch = reinterpret_cast<float*>(gbase + L::kOffXch);
   uint32_t* holder = reinterpret_cast<uint32_t*>(gbase + L::kOffHolder);
   volatile int* abort = reinterpret_cast<volatile int*>(gbase + L::kOffAbort);
 
@@ -199,7 +205,6 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
       mbar_init(bar_s_full + 8 * i, 1);
       mbar_init(bar_p_h0 + 8 * i, kBM);
       mbar_init(bar_p_h1 + 8 * i, kBM);
-      mbar_init(bar_pv_h0 + 8 * i, 1);
     }
     *abort = 0;
     mbar_fence_init();
@@ -257,8 +262,9 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
 #pragma unroll
         for (int k4 = 0; k4 < 4; ++k4) {
           const int kk = 4 * half + k4;
-          umma_ts(tmem + col_o(t), tmem + col_s(t) + kk * 8, sdesc_sw128(v_tile + kk * 2048, kChunkBytes, 1024),
-                  idesc_pv, (acc || kk > 0) ? 1u : 0u);
+          // P of keys [64 h, 64 h + 64) lives in S columns [64 h, 64 h + 32)
+          umma_ts(tmem + col_o(t), tmem + col_s(t) + 64 * half + k4 * 8,
+                  sdesc_sw128(v_tile + kk * 2048, kChunkBytes, 1024), idesc_pv, (acc || kk > 0) ? 1u : 0u);
         }
       };
       // K_j is ring item 2j, V_j item 2j + 1.
@@ -285,7 +291,6 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
           if (p.debug_skip_last_pv && !more) { ok = false; break; }   // the softmax's final wait must expire
           tc_fence_after();
           issue_pv(t, 0, v_tile, j > 0);
-          umma_commit(bar_pv_h0 + 8 * t);
           if (!mbar_wait(bar_p_h1 + 8 * t, j & 1, abort, p.err, p.wait_limit)) { ok = false; break; }
           tc_fence_after();
           issue_pv(t, 1, v_tile, true);
@@ -307,102 +312,111 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
     __syncwarp();
   } else {
     // ------------------------------------------------------------ softmax
-    const int t = warp >> 2;                                      // 0 = tile A, 1 = tile B
+    const int t = warp >> 3;                                      // 0 = tile A, 1 = tile B
+    const int c = (warp >> 2) & 1;                                // key half: columns [64c, 64c + 64)
     if (t == 0 || has_b) {
       const int r = threadIdx.x & 127;                            // query row in the tile
       const uint32_t t_lane = tmem + (static_cast<uint32_t>((warp & 3) * 32) << 16);
       const uint32_t colS = col_s(t), colO = col_o(t);
       const uint32_t bar_s = bar_s_full + 8 * t;
-      const uint32_t bar_ph0 = bar_p_h0 + 8 * t, bar_ph1 = bar_p_h1 + 8 * t, bar_pvh0 = bar_pv_h0 + 8 * t;
+      const uint32_t bar_ph = (c == 0 ? bar_p_h0 : bar_p_h1) + 8 * t;
+      // exchange slots, double-buffered by tile parity: slot(par, group)
+      auto slot = [&](int par, int grp) { return xch + ((par * 2 + t) * 2 + grp) * 128; };
       const float sl2 = p.scale_log2;
       float m_used = -INFINITY;                                  // running max in use (log2 units)
-      float2 l2 = make_float2(0.f, 0.f);                         // row sum, two partial lanes
-      bool ok = true;
-      // O *= a (all 32-bit columns of this lane's O row)
+      float2 l2 = make_float2(0.f, 0.f);                         // this half's row sum, two lanes
+      // O *= a over this group's half of the O columns
       auto rescale_o = [&](float a) {
 #pragma unroll
-        for (int c0 = 0; c0 < D; c0 += 32) {
+        for (int c0 = 0; c0 < D / 2; c0 += 32) {
           uint32_t o[32];
-          tmem_ld_32(t_lane + colO + c0, o);
+          tmem_ld_32(t_lane + colO + c * (D / 2) + c0, o);
 #pragma unroll
-          for (int c = 0; c < 32; ++c) o[c] = __float_as_uint(__uint_as_float(o[c]) * a);
-          tmem_st_32(t_lane + colO + c0, o);
+          for (int k = 0; k < 32; ++k) o[k] = __float_as_uint(__uint_as_float(o[k]) * a);
+          tmem_st_32(t_lane + colO + c * (D / 2) + c0, o);
         }
       };
+      // An expired wait sets the abort flag; the groups then run on over stale
+      // TMEM (in bounds) so that both groups of a tile meet every named barrier.
       for (int j = 0; j < T; ++j) {
-        if (!warp_wait(bar_s, j & 1, abort, p.err, p.wait_limit)) { ok = false; break; }
+        warp_wait(bar_s, j & 1, abort, p.err, p.wait_limit);
         tc_fence_after();
         const int valid = j < n_p ? min(kBN, p.P - j * kBN) : min(kBN, p.G - (j - n_p) * kBN);
-        float x[64];
-        if (j == 0) {
-          load_scores(t_lane + colS, 0, valid, x);
-          float mt = max64(x);
-          load_scores(t_lane + colS + 64, 64, valid, x);
-          mt = fmaxf(mt, max64(x));
-          m_used = mt * sl2;
+        float hm = -INFINITY;
+#pragma unroll
+        for (int q32 = 0; q32 < 2; ++q32) {
+          float x[32];
+          load_scores32(t_lane + colS + 64 * c + 32 * q32, 64 * c + 32 * q32, valid, x);
+          hm = fmaxf(hm, max32(x));
         }
+        // A slot of parity j & 1 is rewritten at tile j + 2 only after both
+        // groups passed tile j + 1's barrier, i.e. after it was read.
+        slot(j & 1, c)[r] = hm * sl2;
+        tile_bar(t);                       // both halves' maxima published
+        const float tm = fmaxf(slot(j & 1, c)[r], slot(j & 1, c ^ 1)[r]);
+        if (j == 0) {
+          m_used = tm;
+        } else if (__any_sync(0xffffffffu, tm > m_used + 8.0f)) {
+          // Same rows, same maxima in both groups: the same decision.  O holds
+          // P V up to tile j-1, complete (S(j) was announced after it).
+          const float m_new = fmaxf(m_used, tm);
+          const float a = ex2_approx(m_used - m_new);
+          m_used = m_new;
+          l2.x *= a;
+          l2.y *= a;
+          rescale_o(a);
+        }
+        const float2 neg_m = make_float2(-m_used, -m_used);
+        const float2 slv = make_float2(sl2, sl2);
+        float2 acc[2] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
 #pragma unroll
-        for (int half = 0; half < 2; ++half) {
-          load_scores(t_lane + colS + 64 * half, 64 * half, valid, x);
-          const float hm = max64(x) * sl2;
-          if (__any_sync(0xffffffffu, hm > m_used + 8.0f)) {
-            const float m_new = fmaxf(m_used, hm);
-            const float a = ex2_approx(m_used - m_new);
-            m_used = m_new;
-            l2.x *= a;
-            l2.y *= a;
-            if (half == 1) {
-              // P V of the first half may already have accumulated into O with
-              // the old max: rescale O once it has.
-              if (!warp_wait(bar_pvh0, j & 1, abort, p.err, p.wait_limit)) { ok = false; break; }
-              tc_fence_after();
-            }
-            // (half 0: O holds P V up to tile j-1, complete -- S(j) was announced after it)
-            rescale_o(a);
-          }
-          const float2 neg_m = make_float2(-m_used, -m_used);
-          const float2 slv = make_float2(sl2, sl2);
-          uint32_t pk[32];
-          float2 acc[2] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
+        for (int q32 = 0; q32 < 2; ++q32) {
+          float x[32];
+          load_scores32(t_lane + colS + 64 * c + 32 * q32, 64 * c + 32 * q32, valid, x);
+          uint32_t pk[16];
 #pragma unroll
-          for (int c = 0; c < 32; ++c) {
-            const float2 y = ffma2(make_float2(x[2 * c], x[2 * c + 1]), slv, neg_m);
+          for (int k = 0; k < 16; ++k) {
+            const float2 y = ffma2(make_float2(x[2 * k], x[2 * k + 1]), slv, neg_m);
             const float p0 = ex2_approx(y.x);
             const float p1 = ex2_approx(y.y);
-            acc[c & 1] = fadd2(acc[c & 1], make_float2(p0, p1));
-            pk[c] = pack_bf16x2(p0, p1);
+            acc[k & 1] = fadd2(acc[k & 1], make_float2(p0, p1));
+            pk[k] = pack_bf16x2(p0, p1);
           }
-          l2 = fadd2(l2, fadd2(acc[0], acc[1]));
-          tmem_st_32(t_lane + colS + 32 * half, pk);     // P half over S columns already read
-          tc_fence_before();
-          mbar_arrive(half == 0 ? bar_ph0 : bar_ph1);
+          // P over this group's own S columns, already read (the second
+          // chunk's S columns [32, 64) stay unwritten until read)
+          tmem_st_16(t_lane + colS + 64 * c + 16 * q32, pk);
         }
-        if (!ok) break;
+        l2 = fadd2(l2, fadd2(acc[0], acc[1]));
+        tc_fence_before();
+        mbar_arrive(bar_ph);
       }
-      const float l_sum = l2.x + l2.y;
-      if (ok && warp_wait(bar_s, T & 1, abort, p.err, p.wait_limit)) {
-        tc_fence_after();
-        const float inv_l = 1.0f / l_sum;
-        const int q = q0 + t * kBM + r;
-        const bool live = q < p.M;
-        __nv_bfloat16* orow = p.out + ((static_cast<size_t>(b) * p.M + q) * p.Hq + h) * D;
+      // epilogue: combine the two halves' row sums, normalise this half of O
+      const bool ok = warp_wait(bar_s, T & 1, abort, p.err, p.wait_limit);
+      tc_fence_after();
+      tile_bar(t);                         // every exchange slot has been read
+      slot(0, c)[r] = l2.x + l2.y;
+      tile_bar(t);
+      const float l_sum = slot(0, c)[r] + slot(0, c ^ 1)[r];
+      const float inv_l = 1.0f / l_sum;
+      const int q = q0 + t * kBM + r;
+      const bool live = ok && q < p.M;
+      __nv_bfloat16* orow = p.out + ((static_cast<size_t>(b) * p.M + q) * p.Hq + h) * D + c * (D / 2);
 #pragma unroll
-        for (int c0 = 0; c0 < D; c0 += 32) {
-          uint32_t o[32];
-          tmem_ld_32(t_lane + colO + c0, o);
-          uint32_t w[16];
+      for (int c0 = 0; c0 < D / 2; c0 += 32) {
+        uint32_t o[32];
+        tmem_ld_32(t_lane + colO + c * (D / 2) + c0, o);
+        uint32_t w[16];
 #pragma unroll
-          for (int c = 0; c < 16; ++c)
-            w[c] = pack_bf16x2(__uint_as_float(o[2 * c]) * inv_l, __uint_as_float(o[2 * c + 1]) * inv_l);
-          if (live) {
-            uint4* dst = reinterpret_cast<uint4*>(orow + c0);
+        for (int k = 0; k < 16; ++k)
+          w[k] = pack_bf16x2(__uint_as_float(o[2 * k]) * inv_l, __uint_as_float(o[2 * k + 1]) * inv_l);
+        if (live) {
+          uint4* dst = reinterpret_cast<uint4*>(orow + c0);
 #pragma unroll
-            for (int v = 0; v < 4; ++v) dst[v] = make_uint4(w[4 * v], w[4 * v + 1], w[4 * v + 2], w[4 * v + 3]);
-          }
+          for (int v = 0; v < 4; ++v) dst[v] = make_uint4(w[4 * v], w[4 * v + 1], w[4 * v + 2], w[4 * v + 3]);
         }
-        if (live && p.lse)
-          p.lse[(static_cast<size_t>(b) * p.Hq + h) * p.M + q] = (m_used + log2f(l_sum)) * 0.69314718055994531f;
       }
+      if (live && c == 0 && p.lse)
+        p.lse[(static_cast<size_t>(b) * p.Hq + h) * p.M + q] = (m_used + log2f(l_sum)) * 0.69314718055994531f;
     }
   }
 
