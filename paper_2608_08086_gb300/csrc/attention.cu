@@ -144,6 +144,26 @@ __device__ __forceinline__ float max32(const float (&x)[32]) {
   return max3f(m[0], m[1], fmaxf(m[2], m[3]));
 }
 
+__device__ __forceinline__ float max64(const float (&x)[64]) {
+  float m[4] = {x[0], x[1], x[2], x[3]};
+#pragma unroll
+  for (int c = 4; c < 64; c += 2) m[(c >> 1) & 3] = max3f(m[(c >> 1) & 3], x[c], x[c + 1]);
+  return max3f(m[0], m[1], fmaxf(m[2], m[3]));
+}
+
+// Loads 64 score columns [c0, c0 + 64) of this lane and masks keys >= valid.
+__device__ __forceinline__ void load_scores64(uint32_t taddr, int c0, int valid, float (&x)[64]) {
+  uint32_t r[64];
+  tmem_ld_64(taddr, r);
+#pragma unroll
+  for (int c = 0; c < 64; ++c) x[c] = __uint_as_float(r[c]);
+  if (valid < c0 + 64) {            // only the last tile of a segment is ragged
+#pragma unroll
+    for (int c = 0; c < 64; ++c)
+      if (c0 + c >= valid) x[c] = -INFINITY;
+  }
+}
+
 // Loads 32 score columns [c0, c0 + 32) of this lane and masks keys >= valid.
 __device__ __forceinline__ void load_scores32(uint32_t taddr, int c0, int valid, float (&x)[32]) {
   uint32_t r[32];
@@ -342,12 +362,11 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
         warp_wait(bar_s, j & 1, abort, p.err, p.wait_limit);
         tc_fence_after();
         const int valid = j < n_p ? min(kBN, p.P - j * kBN) : min(kBN, p.G - (j - n_p) * kBN);
-        float hm = -INFINITY;
-#pragma unroll
-        for (int q32 = 0; q32 < 2; ++q32) {
-          float x[32];
-          load_scores32(t_lane + colS + 64 * c + 32 * q32, 64 * c + 32 * q32, valid, x);
-          hm = fmaxf(hm, max32(x));
+        float hm;
+        {
+          float x[64];
+          load_scores64(t_lane + colS + 64 * c, 64 * c, valid, x);
+          hm = max64(x);
         }
         // A slot of parity j & 1 is rewritten at tile j + 2 only after both
         // groups passed tile j + 1's barrier, i.e. after it was read.
@@ -369,23 +388,25 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
         const float2 neg_m = make_float2(-m_used, -m_used);
         const float2 slv = make_float2(sl2, sl2);
         float2 acc[2] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
+        uint32_t pk[2][16];
 #pragma unroll
         for (int q32 = 0; q32 < 2; ++q32) {
           float x[32];
           load_scores32(t_lane + colS + 64 * c + 32 * q32, 64 * c + 32 * q32, valid, x);
-          uint32_t pk[16];
 #pragma unroll
           for (int k = 0; k < 16; ++k) {
             const float2 y = ffma2(make_float2(x[2 * k], x[2 * k + 1]), slv, neg_m);
             const float p0 = ex2_approx(y.x);
             const float p1 = ex2_approx(y.y);
             acc[k & 1] = fadd2(acc[k & 1], make_float2(p0, p1));
-            pk[k] = pack_bf16x2(p0, p1);
+            pk[q32][k] = pack_bf16x2(p0, p1);
           }
           // P over this group's own S columns, already read (the second
-          // chunk's S columns [32, 64) stay unwritten until read)
-          tmem_st_16(t_lane + colS + 64 * c + 16 * q32, pk);
+          // chunk's S columns [32, 64) stay unwritten until read).  The store
+          // stays in flight while the next chunk is computed.
+          tmem_st_16_async(t_lane + colS + 64 * c + 16 * q32, pk[q32]);
         }
+        tmem_wait_st();
         l2 = fadd2(l2, fadd2(acc[0], acc[1]));
         tc_fence_before();
         mbar_arrive(bar_ph);
