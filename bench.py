@@ -47,6 +47,30 @@ import torch  # noqa: E402
 from paper_2608_08086_gb300 import synth  # noqa: E402
 
 METRIC = "denoise steps/s"
+
+# DRAM traffic per launch (dram__bytes_read.sum + dram__bytes_write.sum) from one
+# ncu capture of the same launch configuration (see profiles/).  A figure is
+# valid only for the kernel source it was captured on: the sha256 prefix of the
+# translation unit is checked at run time and the figure dropped on mismatch.
+MEASURED_TRAFFIC = {
+    # (kernel, workload): {"bytes": per launch, "source": file, "sha16": sha256[:16]}
+}
+
+
+def _source_sha(rel):
+    import hashlib
+    with open(os.path.join(ROOT, rel), "rb") as f:
+        return hashlib.sha256(f.read()).hexdigest()[:16]
+
+
+def measured_traffic(kernel, workload):
+    ent = MEASURED_TRAFFIC.get((kernel, workload))
+    if not ent:
+        return None
+    try:
+        return ent["bytes"] if _source_sha(ent["source"]) == ent["sha16"] else None
+    except OSError:
+        return None
 PEAKS_FALLBACK = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 
 
@@ -208,43 +232,57 @@ def run_e2e(wl, steps, warmup, dist_on, seed=0):
     """The same step through the C ABI with HOST inputs: every step copies its
     inputs (token updates, redrawn Q/K/V rows of every layer, the step's logits,
     and at a refresh the fresh prompt Q/K/V of every layer) from pinned host
-    memory, and reads the scores back."""
+    memory and reads the scores back.  The per-step uploads are double-buffered
+    on a copy stream (step t+2's inputs are uploaded while step t computes);
+    a refresh step's prompt uploads happen in the step, once the rule has fired.
+    The timed region starts before the first upload and issues exactly the
+    uploads of the timed steps."""
     from paper_2608_08086_gb300.trajectory import DeviceTrajectory
-    tr = DeviceTrajectory(wl, seed=seed, mode="archer", source="device", max_steps=warmup + steps + 1)
+    tr = DeviceTrajectory(wl, seed=seed, mode="archer", source="device", max_steps=warmup + steps + 2)
     sh = wl.shape
-    B, P, G, Hq, Hkv, D, L = sh.batch, sh.prompt_len, sh.resp_len, sh.n_heads, sh.n_kv_heads, sh.head_dim, tr.L
-    n = wl.redraws_per_step
-    # host staging buffers (pinned): one layer's worth, copied to every layer
-    h_rows_q = tr.pool["q"][0].cpu().pin_memory()          # [L, B, n, Hq, D]
-    h_rows_k = tr.pool["k"][0].cpu().pin_memory()
-    h_rows_v = tr.pool["v"][0].cpu().pin_memory()
+    B, P, G, L = sh.batch, sh.prompt_len, sh.resp_len, tr.L
+    copy_stream = torch.cuda.Stream()
+    nb = lambda t: t.numel() * t.element_size()  # noqa: E731
+    # host sources (pinned): one step's redraw rows, the logits, one layer's fresh prompt
+    h_rows = {c: tr.pool[c][0].cpu().pin_memory() for c in ("q", "k", "v")}
     h_logits = tr.logits.cpu().pin_memory()
+    h_plan = [(p.cpu().pin_memory(), v.cpu().pin_memory()) for p, v in tr.plan]
     h_q_prompt = tr.q_all[0][:, :P].contiguous().cpu().pin_memory()
     h_k_new = tr.k_new[0].cpu().pin_memory()
     h_v_new = tr.v_new[0].cpu().pin_memory()
     h_scores = torch.empty(3, B * G, dtype=torch.float32).pin_memory()
-    d_rows = {c: torch.empty_like(tr.pool[c][0]) for c in ("q", "k", "v")}
-    plan_host = [(p.cpu().pin_memory(), v.cpu().pin_memory()) for p, v in tr.plan]
-    d_pos = torch.empty_like(tr.plan[0][0])
-    d_new = torch.empty_like(tr.plan[0][1])
-    bytes_in = {"step": 0, "refresh": 0}
+    # device staging, two sets
+    d_rows = [{c: torch.empty_like(tr.pool[c][0]) for c in ("q", "k", "v")} for _ in range(2)]
+    d_logits = [tr.logits, torch.empty_like(tr.logits)]
+    d_plan = [(torch.empty_like(tr.plan[0][0]), torch.empty_like(tr.plan[0][1])) for _ in range(2)]
+    ready = [torch.cuda.Event() for _ in range(2)]
+    consumed = [torch.cuda.Event() for _ in range(2)]
+    for e in consumed:
+        e.record()
 
-    orig_stage = tr._stage_redraw
-    orig_fresh = tr._stage_fresh_prompt
+    def upload(t):
+        slot = t & 1
+        hp, hn = h_plan[(t - 1) % len(h_plan)]
+        with torch.cuda.stream(copy_stream):
+            copy_stream.wait_event(consumed[slot])
+            d_plan[slot][0].copy_(hp, non_blocking=True)
+            d_plan[slot][1].copy_(hn, non_blocking=True)
+            for c in ("q", "k", "v"):
+                d_rows[slot][c].copy_(h_rows[c], non_blocking=True)
+            d_logits[slot].copy_(h_logits, non_blocking=True)
+            ready[slot].record(copy_stream)
 
     def stage_redraw(t):
-        hp, hn = plan_host[(t - 1) % len(plan_host)]
-        d_pos.copy_(hp, non_blocking=True)
-        d_new.copy_(hn, non_blocking=True)
-        for c, h in (("q", h_rows_q), ("k", h_rows_k), ("v", h_rows_v)):
-            d_rows[c].copy_(h, non_blocking=True)
-        tr.logits.copy_(h_logits, non_blocking=True)
+        slot = t & 1
+        torch.cuda.current_stream().wait_event(ready[slot])
+        pos, new = d_plan[slot]
         bidx = torch.arange(B, device=tr.device)[:, None]
-        tr.g[bidx, d_pos] = d_new
-        tr.q_resp[:, bidx, d_pos] = d_rows["q"]
-        tr.q_all[:, bidx, P + d_pos] = d_rows["q"]
-        tr.k_resp[:, bidx, d_pos] = d_rows["k"]
-        tr.v_resp[:, bidx, d_pos] = d_rows["v"]
+        tr.g[bidx, pos] = new
+        tr.q_resp[:, bidx, pos] = d_rows[slot]["q"]
+        tr.q_all[:, bidx, P + pos] = d_rows[slot]["q"]
+        tr.k_resp[:, bidx, pos] = d_rows[slot]["k"]
+        tr.v_resp[:, bidx, pos] = d_rows[slot]["v"]
+        tr.logits = d_logits[slot]
 
     def stage_fresh(t):
         for layer in range(L):
@@ -254,23 +292,30 @@ def run_e2e(wl, steps, warmup, dist_on, seed=0):
 
     tr._stage_redraw = stage_redraw
     tr._stage_fresh_prompt = stage_fresh
-    nb = lambda t: t.numel() * t.element_size()  # noqa: E731
-    per_step_in = (nb(plan_host[0][0]) + nb(plan_host[0][1]) + nb(h_rows_q) + nb(h_rows_k) + nb(h_rows_v)
-                   + nb(h_logits))
+    per_step_in = nb(h_plan[0][0]) + nb(h_plan[0][1]) + sum(nb(h) for h in h_rows.values()) + nb(h_logits)
     per_refresh_in = L * (nb(h_q_prompt) + nb(h_k_new) + nb(h_v_new))
+
+    def run_steps(first, count):
+        upload(first)
+        if count > 1:
+            upload(first + 1)
+        for i in range(count):
+            t = first + i
+            tr.step()
+            h_scores[0].copy_(tr.max_prob, non_blocking=True)
+            h_scores[1].copy_(tr.top1.view(torch.float32), non_blocking=True)
+            h_scores[2].copy_(tr.margin, non_blocking=True)
+            consumed[t & 1].record()
+            if i + 2 < count:
+                upload(t + 2)
+
     tr.build()
-    for _ in range(warmup):
-        tr.step()
-        h_scores[0].copy_(tr.max_prob, non_blocking=True)
+    run_steps(1, warmup)
     barrier(dist_on)
     r0 = tr.n_refresh_steps
     start, end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     start.record()
-    for _ in range(steps):
-        tr.step()
-        h_scores[0].copy_(tr.max_prob, non_blocking=True)
-        h_scores[1].copy_(tr.top1.view(torch.float32), non_blocking=True)
-        h_scores[2].copy_(tr.margin, non_blocking=True)
+    run_steps(warmup + 1, steps)
     end.record()
     barrier(dist_on)
     ms = start.elapsed_time(end)
@@ -279,7 +324,7 @@ def run_e2e(wl, steps, warmup, dist_on, seed=0):
     d2h = B + 3 * B * G * 4      # the refresh flags and the three score vectors
     del tr
     torch.cuda.empty_cache()
-    return {"ms": ms, "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h)}
+    return {"ms": ms, "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h), "overlap": "copy stream"}
 
 
 # ---------------------------------------------------------------------------- oracle (CPU)
@@ -413,13 +458,15 @@ def main():
             tot_flops += fl * k["count"]
             tot_ms += k["total_ms"]
     peak_tf = pk["bf16_tflops_sustained"]
-    achieved = tot_flops / (tot_ms * 1e9) if tot_ms else 0.0
+    # roofline of the dominant kernel: its cached-step launches (one FLOP count)
+    achieved = att["step"]["tflops"] if "step" in att else (tot_flops / (tot_ms * 1e9) if tot_ms else 0.0)
     scoring = None
     if "score" in ks:
         sbytes = tr.B * tr.G * wl.vocab * (2 if wl.logits_dtype == "bf16" else 4)
         gbs = sbytes / (ks["score"]["mean_ms"] * 1e6)
         scoring = {"mean_ms": ks["score"]["mean_ms"], "gbs": gbs, "peak_gbs": pk["hbm_gbs"],
-                   "frac": gbs / pk["hbm_gbs"], "bytes_per_launch": sbytes}
+                   "frac": gbs / pk["hbm_gbs"], "bytes_per_launch": sbytes,
+                   "traffic": measured_traffic("scores", wl.name)}
     del arm, tr
     torch.cuda.empty_cache()
 
@@ -477,9 +524,11 @@ def main():
             "speedup_vs_refresh_every_step": value / eager_value,
             "eager_steps_per_s": eager_value,
             "attention": att,
-            "roofline": {"bound": "tensor", "kernel": "attn_fwd_kernel<128>", "achieved": achieved, "peak": peak_tf,
-                         "unit": "TFLOP/s", "frac": achieved / peak_tf, "traffic": None,
-                         "peak_kind": f"bf16_tflops_sustained ({pk_kind})"},
+            "roofline": {"bound": "tensor", "kernel": "attn_fwd_kernel<128>", "launches": "cached step",
+                         "flops_per_launch": flops_step_launch, "achieved": achieved, "peak": peak_tf,
+                         "unit": "TFLOP/s", "frac": achieved / peak_tf,
+                         "traffic": measured_traffic("attn_step", wl.name),
+                         "peak_kind": f"bf16_tflops_sustained ({pk_kind}; the kernel runs inside a long step)"},
             "scoring": scoring,
             "e2e": e2e,
             "gpu_launches": launches,
