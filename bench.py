@@ -53,14 +53,23 @@ METRIC = "denoise steps/s"
 # valid only for the kernel source it was captured on: the sha256 prefix of the
 # translation unit is checked at run time and the figure dropped on mismatch.
 MEASURED_TRAFFIC = {
-    # (kernel, workload): {"bytes": per launch, "source": file, "sha16": sha256[:16]}
+    # (kernel, workload): DRAM bytes read + written per launch from one ncu capture
+    # (dram__bytes_read.sum + dram__bytes_write.sum), valid only while the kernel's
+    # sources hash to sha16 (sha256 over the listed files, first 16 hex digits).
+    ("attn_step", "gqa_long"): {"bytes": 250989056, "sha16": "84b8b1d2d5f5f3ac",
+                                "sources": ["attention.cu", "archer_device.cuh", "tmem_ldst.cuh"]},
+    ("scores", "gqa_long"): {"bytes": 2496365824, "sha16": "dfcf85f945357c7b",
+                             "sources": ["decode_scores.cu", "archer_device.cuh"]},
 }
 
 
-def _source_sha(rel):
+def _source_sha(files):
     import hashlib
-    with open(os.path.join(ROOT, rel), "rb") as f:
-        return hashlib.sha256(f.read()).hexdigest()[:16]
+    h = hashlib.sha256()
+    for f in files:
+        with open(os.path.join(ROOT, "paper_2608_08086_gb300", "csrc", f), "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()[:16]
 
 
 def measured_traffic(kernel, workload):
@@ -68,9 +77,11 @@ def measured_traffic(kernel, workload):
     if not ent:
         return None
     try:
-        return ent["bytes"] if _source_sha(ent["source"]) == ent["sha16"] else None
+        return ent["bytes"] if _source_sha(ent["sources"]) == ent["sha16"] else None
     except OSError:
         return None
+
+
 PEAKS_FALLBACK = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
 
 
