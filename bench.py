@@ -28,6 +28,7 @@ per rank, no collective on the data path ("scaling": "weak").
 from __future__ import annotations
 
 import argparse
+import dataclasses
 import json
 import math
 import os
@@ -229,6 +230,93 @@ def kernel_only(args, wl):
     return 0
 
 
+def _time_launches(fn, runs, flush=None):
+    """Median (cold: L2 flushed before each launch) and mean back-to-back
+    duration in us of fn's launches, CUDA events on the current stream."""
+    cold = []
+    for _ in range(runs):
+        if flush is not None:
+            flush.add_(1)
+        s, e = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        s.record()
+        fn()
+        e.record()
+        e.synchronize()
+        cold.append(s.elapsed_time(e) * 1e3)
+    s, e = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    s.record()
+    for _ in range(runs):
+        fn()
+    e.record()
+    e.synchronize()
+    return statistics.median(cold), s.elapsed_time(e) * 1e3 / runs
+
+
+def _attn_pair(sh, dev, runs, flush):
+    """Cached step and refresh of one layer of shape sh: times and TFLOP/s."""
+    from paper_2608_08086_gb300 import archer as A
+    B, P, G, Hq, Hkv, D = sh.batch, sh.prompt_len, sh.resp_len, sh.n_heads, sh.n_kv_heads, sh.head_dim
+    d = synth.device_attn_inputs(sh, dev, seed=0)
+    shape = A.make_shape(B, P, G, Hq, Hkv, D)
+    q = d["q_all"][:, P:].contiguous()
+    out_g = torch.empty(B, G, Hq, D, dtype=torch.bfloat16, device=dev)
+    out_n = torch.empty(B, P + G, Hq, D, dtype=torch.bfloat16, device=dev)
+    step = lambda: A.archer_attn_step(shape, q, d["k_cache"], d["v_cache"], d["k_resp"], d["v_resp"], out_g)  # noqa: E731
+    refresh = lambda: A.archer_prompt_refresh(shape, d["q_all"], d["k_prompt"], d["v_prompt"], d["k_resp"],  # noqa: E731
+                                              d["v_resp"], out_n, None, d["k_prompt"], d["v_prompt"])
+    for _ in range(3):
+        step()
+        refresh()
+    torch.cuda.synchronize()
+    N = P + G
+    res = {}
+    for name, fn, M in (("step", step, G), ("refresh", refresh, N)):
+        cold, b2b = _time_launches(fn, runs, flush)
+        fl = 4.0 * B * Hq * M * N * D
+        res[name] = {"cold_us": cold, "b2b_us": b2b, "gflop": fl / 1e9, "tflops_cold": fl / cold / 1e6,
+                     "tflops_b2b": fl / b2b / 1e6}
+    A.archer_check_device()
+    res["refresh_over_step"] = res["refresh"]["cold_us"] / res["step"]["cold_us"]
+    res["ideal_ratio_N_over_G"] = N / G
+    return res
+
+
+def sweep(args):
+    """Per-configuration measurements (one JSON line each): the LLaDA-shaped
+    layer (B1, 32 = 32 heads, D128, P512, G256), decoder scoring on
+    [4 x 256 x 126464] bf16, and the prompt-length sweep G = 256,
+    P = 128 ... 2048 with LLaDA heads (cached step vs refresh of one layer).
+    "cold" launches follow a 256 MB L2-flushing write; "b2b" is back to back."""
+    from paper_2608_08086_gb300 import archer as A
+    dev = torch.device("cuda")
+    pk, pk_kind = peaks()
+    flush = torch.zeros(64 << 20, dtype=torch.float32, device=dev)     # 256 MB > L2
+    runs = max(args.launches, 20)
+    wl = synth.WORKLOADS["llada_layer"]
+    print(json.dumps({"sweep": "llada_layer", "shape": dataclasses.asdict(wl.shape), "runs": runs,
+                      **_attn_pair(wl.shape, dev, runs, flush)}), flush=True)
+    wl = synth.WORKLOADS["scoring"]
+    rows = wl.logits_rows
+    z = synth.device_logits(rows, wl.vocab, dev, seed=0, std=wl.logits_std, boost_max=wl.logits_boost)
+    mp = torch.empty(rows, dtype=torch.float32, device=dev)
+    t1 = torch.empty(rows, dtype=torch.int32, device=dev)
+    mg = torch.empty(rows, dtype=torch.float32, device=dev)
+    ws = A.scores_workspace(rows, wl.vocab, dev)
+    fn = lambda: A.archer_decode_scores(z, mp, t1, mg, workspace=ws)  # noqa: E731
+    for _ in range(3):
+        fn()
+    cold, b2b = _time_launches(fn, runs, flush)
+    nbytes = rows * wl.vocab * 2
+    print(json.dumps({"sweep": "scoring", "rows": rows, "vocab": wl.vocab, "bytes": nbytes, "cold_us": cold,
+                      "b2b_us": b2b, "gbs_cold": nbytes / cold / 1e3, "frac_cold": nbytes / cold / 1e3 / pk["hbm_gbs"],
+                      "peak_gbs": pk["hbm_gbs"], "peak_kind": pk_kind}), flush=True)
+    for P in (128, 256, 512, 1024, 2048):
+        sh = synth.AttnShape(1, P, 256, 32, 32, 128)
+        print(json.dumps({"sweep": "prompt_len", "P": P, "G": 256, "runs": runs,
+                          **_attn_pair(sh, dev, runs, flush)}), flush=True)
+    return 0
+
+
 def kernel_stats(tr):
     """Mean durations (ms) and counts of the attention / scoring launches."""
     by = {}
@@ -245,7 +333,8 @@ def run_e2e(wl, steps, warmup, dist_on, seed=0):
     and at a refresh the fresh prompt Q/K/V of every layer) from pinned host
     memory and reads the scores back.  The per-step uploads are double-buffered
     on a copy stream (step t+2's inputs are uploaded while step t computes);
-    a refresh step's prompt uploads happen in the step, once the rule has fired.
+    a refresh step's prompt uploads start once the rule has fired, layer by
+    layer on a second copy stream, each layer's refresh waiting for its own.
     The timed region starts before the first upload and issues exactly the
     uploads of the timed steps."""
     from paper_2608_08086_gb300.trajectory import DeviceTrajectory
@@ -295,11 +384,22 @@ def run_e2e(wl, steps, warmup, dist_on, seed=0):
         tr.v_resp[:, bidx, pos] = d_rows[slot]["v"]
         tr.logits = d_logits[slot]
 
+    fresh_stream = torch.cuda.Stream()
+    layer_ready = [torch.cuda.Event() for _ in range(L)]
+    tr.layer_ready = layer_ready
+
     def stage_fresh(t):
-        for layer in range(L):
-            tr.q_all[layer][:, :P].copy_(h_q_prompt, non_blocking=True)
-            tr.k_new[layer].copy_(h_k_new, non_blocking=True)
-            tr.v_new[layer].copy_(h_v_new, non_blocking=True)
+        # Per-layer uploads on their own stream: layer l's refresh waits only for
+        # its own prompt Q/K/V, so later layers' copies overlap earlier layers' work.
+        here = torch.cuda.Event()
+        here.record()
+        with torch.cuda.stream(fresh_stream):
+            fresh_stream.wait_event(here)
+            for layer in range(L):
+                tr.q_all[layer][:, :P].copy_(h_q_prompt, non_blocking=True)
+                tr.k_new[layer].copy_(h_k_new, non_blocking=True)
+                tr.v_new[layer].copy_(h_v_new, non_blocking=True)
+                layer_ready[layer].record(fresh_stream)
 
     tr._stage_redraw = stage_redraw
     tr._stage_fresh_prompt = stage_fresh
@@ -335,7 +435,7 @@ def run_e2e(wl, steps, warmup, dist_on, seed=0):
     d2h = B + 3 * B * G * 4      # the refresh flags and the three score vectors
     del tr
     torch.cuda.empty_cache()
-    return {"ms": ms, "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h), "overlap": "copy stream"}
+    return {"ms": ms, "h2d_bytes_per_step": int(h2d), "d2h_bytes_per_step": int(d2h), "overlap": "copy streams (per-step double buffer; per-layer refresh uploads)"}
 
 
 # ---------------------------------------------------------------------------- oracle (CPU)
@@ -420,17 +520,19 @@ def main():
     ap.add_argument("--kernel-only", choices=["attn_step", "attn_refresh", "scores"], default=None,
                     help="run only a few launches of one kernel (for profiler captures)")
     ap.add_argument("--launches", type=int, default=3)
+    ap.add_argument("--sweep", action="store_true",
+                    help="per-configuration measurements (LLaDA layer, scoring, prompt-length sweep)")
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3)
     wl = synth.WORKLOADS[args.workload]
 
     if args.impl == "reference":
         return reference_arm(args, wl)
-    if args.kernel_only:
+    if args.kernel_only or args.sweep:
         torch.cuda.set_device(int(os.environ.get("LOCAL_RANK", "0")))
         from paper_2608_08086_gb300 import build as Bld
         Bld.build()
-        return kernel_only(args, wl)
+        return sweep(args) if args.sweep else kernel_only(args, wl)
 
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))

@@ -19,12 +19,16 @@
 //              2^8, rescaling l and each group's half of O).  Each group writes
 //              its half of P (bf16 pairs) over the first 32 of its own 64 S
 //              columns and hands it to the MMA warp at once.
-//   warp 16    TMA producer: Q_A, Q_B once, then K_0, V_0, K_1, V_1, ... tiles
-//              of 128 keys through one 4-slot ring.
+//   warp 16    TMA producer: Q_A, Q_B once, then pairs (V_{u-1}, K_u) of
+//              128-key tiles (u = 0 .. T; the first pair holds K_0 only, the
+//              last V_{T-1} only) through two pair slots, one full and one
+//              empty barrier per pair.
 //   warp 17    MMA issuer (one thread), per K/V tile j:
-//                PV_A(j) in two halves, QK_A(j+1), PV_B(j) in two halves, QK_B(j+1)
+//                PV_A(j), QK_A(j+1), PV_B(j), QK_B(j+1)
 //              so the tensor pipe works on one tile while the other tile's
-//              softmax runs.  tcgen05.mma executes in issue order, so QK_X(j+1)
+//              softmax runs.  The issuing thread waits on three barriers and
+//              commits three times per tile j: every wait or commit between two
+//              MMA batches leaves the tensor pipe idle.  tcgen05.mma executes in issue order, so QK_X(j+1)
 //              overwrites S_X only after PV_X(j) has read P_X(j), and the commit
 //              that announces S_X(j+1) also covers PV_X(j): when the softmax sees
 //              S_X(j+1), O_X is stable and may be rescaled without a wait.
@@ -71,12 +75,12 @@ template <int D>
 struct Layout {
   static constexpr int kChunks = D / 64;                    // 128-byte column chunks
   static constexpr uint32_t kTile = kChunks * kChunkBytes;  // one 128-row tile of D bf16
-  static constexpr int kSlots = 4;                          // K/V ring: item 2j = K_j, 2j+1 = V_j
+  static constexpr int kSlots = 2;                          // pair slots: [V tile | K tile]
   static constexpr uint32_t kOffQ = 0;                      // Q_A, Q_B
   static constexpr uint32_t kOffKV = kOffQ + 2 * kTile;
-  static constexpr uint32_t kOffBar = kOffKV + kSlots * kTile;
-  // q_full, full[slots], empty[slots], s_full[2], p_half0[2], p_half1[2]
-  static constexpr int kBars = 1 + 2 * kSlots + 6;
+  static constexpr uint32_t kOffBar = kOffKV + kSlots * 2 * kTile;
+  // q_full, full[slots], empty[slots], s_full[2], p_full[2]
+  static constexpr int kBars = 1 + 2 * kSlots + 4;
   static constexpr uint32_t kOffXch = kOffBar + 8 * kBars;  // [tile parity][tile][half][row] floats
   static constexpr uint32_t kOffHolder = kOffXch + 2 * 2 * 2 * 128 * 4;
   static constexpr uint32_t kOffAbort = kOffHolder + 4;
@@ -208,8 +212,7 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
   const uint32_t bar_full = bars + 8;                           // + 8 * slot
   const uint32_t bar_empty = bar_full + 8 * L::kSlots;          // + 8 * slot
   const uint32_t bar_s_full = bar_empty + 8 * L::kSlots;        // + 8 * tile (A = 0, B = 1)
-  const uint32_t bar_p_h0 = bar_s_full + 16;                    // + 8 * tile: first half of P written
-  const uint32_t bar_p_h1 = bar_p_h0 + 16;                      // + 8 * tile: second half of P written
+  const uint32_t bar_p_full = bar_s_full + 16;                  // + 8 * tile: both halves of P written
   float* xch = reinterpret_cast<float*>(gbase + L::kOffXch);
   uint32_t* holder = reinterpret_cast<uint32_t*>(gbase + L::kOffHolder);
   volatile int* abort = reinterpret_cast<volatile int*>(gbase + L::kOffAbort);
@@ -223,8 +226,7 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
     }
     for (int i = 0; i < 2; ++i) {
       mbar_init(bar_s_full + 8 * i, 1);
-      mbar_init(bar_p_h0 + 8 * i, kBM);
-      mbar_init(bar_p_h1 + 8 * i, kBM);
+      mbar_init(bar_p_full + 8 * i, 2 * kBM);
     }
     *abort = 0;
     mbar_fence_init();
@@ -248,17 +250,21 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
       for (int t = 0; t < (has_b ? 2 : 1); ++t)
         for (int c = 0; c < L::kChunks; ++c)
           tma_load_4d(sQ + t * L::kTile + c * kChunkBytes, &tmQ, bar_q_full, c * 64, h, q0 + t * kBM, b);
-      for (int item = 0; item < 2 * T; ++item) {
-        const int j = item >> 1;
-        const bool is_v = item & 1;
-        const bool in_prompt = j < n_p;
-        const int row = in_prompt ? j * kBN : (j - n_p) * kBN;
-        const int slot = item % L::kSlots, use = item / L::kSlots;
+      // pair u = (V_{u-1}, K_u) into pair slot u & 1: [V tile | K tile]
+      for (int u = 0; u <= T; ++u) {
+        const int slot = u & 1, use = u >> 1;
         if (use > 0 && !mbar_wait(bar_empty + 8 * slot, (use - 1) & 1, abort, p.err, p.wait_limit)) break;
-        mbar_arrive_expect_tx(bar_full + 8 * slot, L::kTile);
-        const CUtensorMap* map = in_prompt ? (is_v ? mVp : mKp) : (is_v ? &tmVg : &tmKg);
-        for (int c = 0; c < L::kChunks; ++c)
-          tma_load_4d(sKV + slot * L::kTile + c * kChunkBytes, map, bar_full + 8 * slot, c * 64, kvh, row, b);
+        const bool has_v = u >= 1, has_k = u < T;
+        mbar_arrive_expect_tx(bar_full + 8 * slot, (has_v && has_k ? 2 : 1) * L::kTile);
+        for (int part = has_v ? 0 : 1; part < (has_k ? 2 : 1); ++part) {
+          const int j = part == 0 ? u - 1 : u;
+          const bool in_prompt = j < n_p;
+          const int row = in_prompt ? j * kBN : (j - n_p) * kBN;
+          const CUtensorMap* map = in_prompt ? (part == 0 ? mVp : mKp) : (part == 0 ? &tmVg : &tmKg);
+          const uint32_t dst = sKV + (2 * slot + part) * L::kTile;
+          for (int c = 0; c < L::kChunks; ++c)
+            tma_load_4d(dst + c * kChunkBytes, map, bar_full + 8 * slot, c * 64, kvh, row, b);
+        }
       }
     }
     __syncwarp();
@@ -277,56 +283,41 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
                   idesc_qk, kk > 0 ? 1u : 0u);
         }
       };
-      // P V over keys [64 * half, 64 * half + 64) of the tile (4 MMAs of K = 16).
-      auto issue_pv = [&](int t, int half, uint32_t v_tile, bool acc) {
+      // P V over the tile's 128 keys (8 MMAs of K = 16); P of keys
+      // [64 h, 64 h + 64) lives in S columns [64 h, 64 h + 32).
+      auto issue_pv = [&](int t, uint32_t v_tile, bool acc) {
 #pragma unroll
-        for (int k4 = 0; k4 < 4; ++k4) {
-          const int kk = 4 * half + k4;
-          // P of keys [64 h, 64 h + 64) lives in S columns [64 h, 64 h + 32)
-          umma_ts(tmem + col_o(t), tmem + col_s(t) + 64 * half + k4 * 8,
+        for (int kk = 0; kk < 8; ++kk)
+          umma_ts(tmem + col_o(t), tmem + col_s(t) + 64 * (kk >> 2) + (kk & 3) * 8,
                   sdesc_sw128(v_tile + kk * 2048, kChunkBytes, 1024), idesc_pv, (acc || kk > 0) ? 1u : 0u);
-        }
       };
-      // K_j is ring item 2j, V_j item 2j + 1.
-      auto slot_of = [](int item) { return item % L::kSlots; };
-      auto phase_of = [](int item) { return static_cast<uint32_t>(item / L::kSlots) & 1u; };
+      auto v_tile_of = [&](int u) { return sKV + 2 * (u & 1) * L::kTile; };
+      auto k_tile_of = [&](int u) { return sKV + (2 * (u & 1) + 1) * L::kTile; };
+      auto phase_of = [](int u) { return static_cast<uint32_t>(u >> 1) & 1u; };
       bool ok = mbar_wait(bar_q_full, 0, abort, p.err, p.wait_limit) &&
-                mbar_wait(bar_full + 8 * slot_of(0), phase_of(0), abort, p.err, p.wait_limit);
+                mbar_wait(bar_full, phase_of(0), abort, p.err, p.wait_limit);
       if (ok) {
         tc_fence_after();
         for (int t = 0; t < n_tiles; ++t) {
-          issue_qk(t, sKV + slot_of(0) * L::kTile);
+          issue_qk(t, k_tile_of(0));
           umma_commit(bar_s_full + 8 * t);
         }
-        umma_commit(bar_empty + 8 * slot_of(0));
+        umma_commit(bar_empty);               // pair 0 (K_0) read
       }
       for (int j = 0; ok && j < T; ++j) {
         const bool more = j + 1 < T;
-        const int v_item = 2 * j + 1, k_item = 2 * j + 2;
-        const uint32_t v_tile = sKV + slot_of(v_item) * L::kTile;
-        const uint32_t k_tile = sKV + slot_of(k_item) * L::kTile;
-        if (!mbar_wait(bar_full + 8 * slot_of(v_item), phase_of(v_item), abort, p.err, p.wait_limit)) break;
+        const int u = j + 1;                  // pair (V_j, K_{j+1})
+        if (!mbar_wait(bar_full + 8 * (u & 1), phase_of(u), abort, p.err, p.wait_limit)) break;
         for (int t = 0; t < n_tiles; ++t) {
-          if (!mbar_wait(bar_p_h0 + 8 * t, j & 1, abort, p.err, p.wait_limit)) { ok = false; break; }
+          if (!mbar_wait(bar_p_full + 8 * t, j & 1, abort, p.err, p.wait_limit)) { ok = false; break; }
           if (p.debug_skip_last_pv && !more) { ok = false; break; }   // the softmax's final wait must expire
           tc_fence_after();
-          issue_pv(t, 0, v_tile, j > 0);
-          if (!mbar_wait(bar_p_h1 + 8 * t, j & 1, abort, p.err, p.wait_limit)) { ok = false; break; }
-          tc_fence_after();
-          issue_pv(t, 1, v_tile, true);
-          if (more) {
-            if (t == 0 && !mbar_wait(bar_full + 8 * slot_of(k_item), phase_of(k_item), abort, p.err, p.wait_limit)) {
-              ok = false;
-              break;
-            }
-            tc_fence_after();
-            issue_qk(t, k_tile);
-          }
+          issue_pv(t, v_tile_of(u), j > 0);
+          if (more) issue_qk(t, k_tile_of(u));
           umma_commit(bar_s_full + 8 * t);   // S_t(j+1) ready -- or, after the last tile, O_t final
         }
         if (!ok) break;
-        umma_commit(bar_empty + 8 * slot_of(v_item));
-        if (more) umma_commit(bar_empty + 8 * slot_of(k_item));
+        umma_commit(bar_empty + 8 * (u & 1));
       }
     }
     __syncwarp();
@@ -339,7 +330,7 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
       const uint32_t t_lane = tmem + (static_cast<uint32_t>((warp & 3) * 32) << 16);
       const uint32_t colS = col_s(t), colO = col_o(t);
       const uint32_t bar_s = bar_s_full + 8 * t;
-      const uint32_t bar_ph = (c == 0 ? bar_p_h0 : bar_p_h1) + 8 * t;
+      const uint32_t bar_ph = bar_p_full + 8 * t;
       // exchange slots, double-buffered by tile parity: slot(par, group)
       auto slot = [&](int par, int grp) { return xch + ((par * 2 + t) * 2 + grp) * 128; };
       const float sl2 = p.scale_log2;

@@ -57,6 +57,7 @@ class DeviceTrajectory:
         self.t = -1
         self.attn_events = []          # (start, end, kind) CUDA events around attention launches
         self.time_attention = False
+        self.layer_ready = None        # optional per-layer CUDA events a refresh layer waits on
         self._alloc()
 
     # ------------------------------------------------------------------ setup
@@ -133,6 +134,8 @@ class DeviceTrajectory:
         outs = []
         for layer in range(self.L):
             if refresh:
+                if self.layer_ready is not None:
+                    torch.cuda.current_stream().wait_event(self.layer_ready[layer])
                 self._timed("refresh", lambda: A.archer_prompt_refresh(
                     self.shape, self.q_all[layer], self.k_new[layer], self.v_new[layer], self.k_resp[layer],
                     self.v_resp[layer], self.out_full, None, self.k_cache[layer], self.v_cache[layer],
