@@ -10,28 +10,30 @@
 //
 // One CTA = two 128-row query tiles (A and B) of one (b, h) sharing every K/V
 // tile; 18 warps:
-//   warps 0-15 softmax: four warpgroups, (tile A, keys 0-63), (A, 64-127),
-//              (B, 0-63), (B, 64-127).  Thread t of a warpgroup owns query row
-//              t (TMEM lane t) for its 64 key columns.  The two groups of a
-//              tile exchange their row maxima through shared memory (a named
-//              barrier per tile); exponentials use the running max in use,
-//              raised lazily (only when the tile max exceeds it by more than
-//              2^8, rescaling l and each group's half of O).  Each group writes
-//              its half of P (bf16 pairs) over the first 32 of its own 64 S
-//              columns and hands it to the MMA warp at once.
-//   warp 16    TMA producer: Q_A, Q_B once, then pairs (V_{u-1}, K_u) of
+//   warp 0     MMA issuer: the warp waits together, lane 0 issues.  Per K/V
+//              tile j: PV_A(j), QK_A(j+1), PV_B(j), QK_B(j+1), so the tensor
+//              pipe works on one tile while the other tile's softmax runs.  It
+//              waits on three barriers and commits three times per tile j:
+//              every wait or commit between two MMA batches idles the tensor
+//              pipe.  tcgen05.mma executes in issue order, so QK_X(j+1)
+//              overwrites S_X only after PV_X(j) has read P_X(j), and the
+//              commit that announces S_X(j+1) also covers PV_X(j): when the
+//              softmax sees S_X(j+1), O_X is stable and may be rescaled without
+//              a wait.
+//   warp 1     TMA producer: Q_A, Q_B once, then pairs (V_{u-1}, K_u) of
 //              128-key tiles (u = 0 .. T; the first pair holds K_0 only, the
 //              last V_{T-1} only) through two pair slots, one full and one
 //              empty barrier per pair.
-//   warp 17    MMA issuer (one thread), per K/V tile j:
-//                PV_A(j), QK_A(j+1), PV_B(j), QK_B(j+1)
-//              so the tensor pipe works on one tile while the other tile's
-//              softmax runs.  The issuing thread waits on three barriers and
-//              commits three times per tile j: every wait or commit between two
-//              MMA batches leaves the tensor pipe idle.  tcgen05.mma executes in issue order, so QK_X(j+1)
-//              overwrites S_X only after PV_X(j) has read P_X(j), and the commit
-//              that announces S_X(j+1) also covers PV_X(j): when the softmax sees
-//              S_X(j+1), O_X is stable and may be rescaled without a wait.
+//   warps 2-17 softmax: four groups of four consecutive warps, (tile A, keys
+//              0-63), (A, 64-127), (B, 0-63), (B, 64-127).  Warp w reaches TMEM
+//              lanes 32 (w % 4) .. 32 (w % 4) + 31, so lane i of warp w owns
+//              query row 32 (w % 4) + i for its 64 key columns, read from TMEM
+//              once per tile.  The two groups of a tile exchange their row
+//              maxima through shared memory (a named barrier per tile);
+//              exponentials use the running max in use, raised lazily (only
+//              when the tile max exceeds it by more than 2^8, rescaling l and
+//              each group's half of O).  Each group writes its half of P (bf16
+//              pairs) over the first 32 of its own 64 S columns.
 // TMEM (512 columns): S_A [0,128) S_B [128,256) O_A [256,256+D) O_B [384,384+D).
 // Every hand-off is an mbarrier; every wait is bounded (archer_device.cuh).
 
@@ -52,7 +54,7 @@ namespace {
 constexpr int kBM = 128;          // query rows per tile (tcgen05 M)
 constexpr int kBN = 128;          // keys per KV tile (N of Q K^T, K of P V)
 constexpr int kThreads = 576;     // 4 softmax warpgroups + producer warp + MMA warp
-constexpr int kWarpProducer = 16, kWarpMma = 17;
+constexpr int kWarpMma = 0, kWarpProducer = 1, kWarpSoftmax0 = 2;
 constexpr uint32_t kTmemCols = 512;
 // TMEM columns of tile t's S (P is written over its first 64 columns) and O.
 __host__ __device__ constexpr uint32_t col_s(int t) { return 128u * static_cast<uint32_t>(t); }
@@ -141,13 +143,6 @@ __device__ __forceinline__ float2 fadd2(float2 a, float2 b) {
   return d;
 }
 
-__device__ __forceinline__ float max32(const float (&x)[32]) {
-  float m[4] = {x[0], x[1], x[2], x[3]};
-#pragma unroll
-  for (int c = 4; c < 32; c += 2) m[(c >> 1) & 3] = max3f(m[(c >> 1) & 3], x[c], x[c + 1]);
-  return max3f(m[0], m[1], fmaxf(m[2], m[3]));
-}
-
 __device__ __forceinline__ float max64(const float (&x)[64]) {
   float m[4] = {x[0], x[1], x[2], x[3]};
 #pragma unroll
@@ -164,19 +159,6 @@ __device__ __forceinline__ void load_scores64(uint32_t taddr, int c0, int valid,
   if (valid < c0 + 64) {            // only the last tile of a segment is ragged
 #pragma unroll
     for (int c = 0; c < 64; ++c)
-      if (c0 + c >= valid) x[c] = -INFINITY;
-  }
-}
-
-// Loads 32 score columns [c0, c0 + 32) of this lane and masks keys >= valid.
-__device__ __forceinline__ void load_scores32(uint32_t taddr, int c0, int valid, float (&x)[32]) {
-  uint32_t r[32];
-  tmem_ld_32(taddr, r);
-#pragma unroll
-  for (int c = 0; c < 32; ++c) x[c] = __uint_as_float(r[c]);
-  if (valid < c0 + 32) {            // only the last tile of a segment is ragged
-#pragma unroll
-    for (int c = 0; c < 32; ++c)
       if (c0 + c >= valid) x[c] = -INFINITY;
   }
 }
@@ -240,20 +222,25 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
   tc_fence_after();
   const uint32_t tmem = *holder;
 
+  const bool lane0 = (threadIdx.x & 31) == 0;
   if (warp == kWarpProducer) {
     // ------------------------------------------------------------ producer
-    if (elect_lane0()) {
-      const CUtensorMap* mKp = refresh ? &tmKpR : &tmKpC;
-      const CUtensorMap* mVp = refresh ? &tmVpR : &tmVpC;
+    // The whole warp runs the loop and waits (warp-uniform); lane 0 issues.
+    const CUtensorMap* mKp = refresh ? &tmKpR : &tmKpC;
+    const CUtensorMap* mVp = refresh ? &tmVpR : &tmVpC;
+    if (lane0) {
       tma_prefetch_map(&tmQ);
       mbar_arrive_expect_tx(bar_q_full, has_b ? 2 * L::kTile : L::kTile);
       for (int t = 0; t < (has_b ? 2 : 1); ++t)
         for (int c = 0; c < L::kChunks; ++c)
           tma_load_4d(sQ + t * L::kTile + c * kChunkBytes, &tmQ, bar_q_full, c * 64, h, q0 + t * kBM, b);
-      // pair u = (V_{u-1}, K_u) into pair slot u & 1: [V tile | K tile]
-      for (int u = 0; u <= T; ++u) {
-        const int slot = u & 1, use = u >> 1;
-        if (use > 0 && !mbar_wait(bar_empty + 8 * slot, (use - 1) & 1, abort, p.err, p.wait_limit)) break;
+    }
+    __syncwarp();
+    // pair u = (V_{u-1}, K_u) into pair slot u & 1: [V tile | K tile]
+    for (int u = 0; u <= T; ++u) {
+      const int slot = u & 1, use = u >> 1;
+      if (use > 0 && !warp_wait(bar_empty + 8 * slot, (use - 1) & 1, abort, p.err, p.wait_limit)) break;
+      if (lane0) {
         const bool has_v = u >= 1, has_k = u < T;
         mbar_arrive_expect_tx(bar_full + 8 * slot, (has_v && has_k ? 2 : 1) * L::kTile);
         for (int part = has_v ? 0 : 1; part < (has_k ? 2 : 1); ++part) {
@@ -266,37 +253,39 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
             tma_load_4d(dst + c * kChunkBytes, map, bar_full + 8 * slot, c * 64, kvh, row, b);
         }
       }
+      __syncwarp();
     }
-    __syncwarp();
   } else if (warp == kWarpMma) {
     // ------------------------------------------------------------ MMA issuer
-    if (elect_lane0()) {
-      constexpr uint32_t idesc_qk = idesc_bf16_f32(kBM, kBN, 0, 0);
-      constexpr uint32_t idesc_pv = idesc_bf16_f32(kBM, D, 0, 1);
-      const int n_tiles = has_b ? 2 : 1;
-      auto issue_qk = [&](int t, uint32_t k_tile) {
-        const uint32_t q_tile = sQ + t * L::kTile;
+    // The whole warp runs the loop and waits (warp-uniform); lane 0 issues
+    // every MMA and commit, so the warp never runs diverged for long.
+    constexpr uint32_t idesc_qk = idesc_bf16_f32(kBM, kBN, 0, 0);
+    constexpr uint32_t idesc_pv = idesc_bf16_f32(kBM, D, 0, 1);
+    const int n_tiles = has_b ? 2 : 1;
+    auto issue_qk = [&](int t, uint32_t k_tile) {
+      const uint32_t q_tile = sQ + t * L::kTile;
 #pragma unroll
-        for (int kk = 0; kk < D / 16; ++kk) {
-          const uint32_t off = (kk >> 2) * kChunkBytes + (kk & 3) * 32;
-          umma_ss(tmem + col_s(t), sdesc_sw128(q_tile + off, 16, 1024), sdesc_sw128(k_tile + off, 16, 1024),
-                  idesc_qk, kk > 0 ? 1u : 0u);
-        }
-      };
-      // P V over the tile's 128 keys (8 MMAs of K = 16); P of keys
-      // [64 h, 64 h + 64) lives in S columns [64 h, 64 h + 32).
-      auto issue_pv = [&](int t, uint32_t v_tile, bool acc) {
+      for (int kk = 0; kk < D / 16; ++kk) {
+        const uint32_t off = (kk >> 2) * kChunkBytes + (kk & 3) * 32;
+        umma_ss(tmem + col_s(t), sdesc_sw128(q_tile + off, 16, 1024), sdesc_sw128(k_tile + off, 16, 1024),
+                idesc_qk, kk > 0 ? 1u : 0u);
+      }
+    };
+    // P V over the tile's 128 keys (8 MMAs of K = 16); P of keys
+    // [64 h, 64 h + 64) lives in S columns [64 h, 64 h + 32).
+    auto issue_pv = [&](int t, uint32_t v_tile, bool acc) {
 #pragma unroll
-        for (int kk = 0; kk < 8; ++kk)
-          umma_ts(tmem + col_o(t), tmem + col_s(t) + 64 * (kk >> 2) + (kk & 3) * 8,
-                  sdesc_sw128(v_tile + kk * 2048, kChunkBytes, 1024), idesc_pv, (acc || kk > 0) ? 1u : 0u);
-      };
-      auto v_tile_of = [&](int u) { return sKV + 2 * (u & 1) * L::kTile; };
-      auto k_tile_of = [&](int u) { return sKV + (2 * (u & 1) + 1) * L::kTile; };
-      auto phase_of = [](int u) { return static_cast<uint32_t>(u >> 1) & 1u; };
-      bool ok = mbar_wait(bar_q_full, 0, abort, p.err, p.wait_limit) &&
-                mbar_wait(bar_full, phase_of(0), abort, p.err, p.wait_limit);
-      if (ok) {
+      for (int kk = 0; kk < 8; ++kk)
+        umma_ts(tmem + col_o(t), tmem + col_s(t) + 64 * (kk >> 2) + (kk & 3) * 8,
+                sdesc_sw128(v_tile + kk * 2048, kChunkBytes, 1024), idesc_pv, (acc || kk > 0) ? 1u : 0u);
+    };
+    auto v_tile_of = [&](int u) { return sKV + 2 * (u & 1) * L::kTile; };
+    auto k_tile_of = [&](int u) { return sKV + (2 * (u & 1) + 1) * L::kTile; };
+    auto phase_of = [](int u) { return static_cast<uint32_t>(u >> 1) & 1u; };
+    bool ok = warp_wait(bar_q_full, 0, abort, p.err, p.wait_limit) &&
+              warp_wait(bar_full, phase_of(0), abort, p.err, p.wait_limit);
+    if (ok) {
+      if (lane0) {
         tc_fence_after();
         for (int t = 0; t < n_tiles; ++t) {
           issue_qk(t, k_tile_of(0));
@@ -304,29 +293,34 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
         }
         umma_commit(bar_empty);               // pair 0 (K_0) read
       }
-      for (int j = 0; ok && j < T; ++j) {
-        const bool more = j + 1 < T;
-        const int u = j + 1;                  // pair (V_j, K_{j+1})
-        if (!mbar_wait(bar_full + 8 * (u & 1), phase_of(u), abort, p.err, p.wait_limit)) break;
-        for (int t = 0; t < n_tiles; ++t) {
-          if (!mbar_wait(bar_p_full + 8 * t, j & 1, abort, p.err, p.wait_limit)) { ok = false; break; }
-          if (p.debug_skip_last_pv && !more) { ok = false; break; }   // the softmax's final wait must expire
+      __syncwarp();
+    }
+    for (int j = 0; ok && j < T; ++j) {
+      const bool more = j + 1 < T;
+      const int u = j + 1;                    // pair (V_j, K_{j+1})
+      if (!warp_wait(bar_full + 8 * (u & 1), phase_of(u), abort, p.err, p.wait_limit)) break;
+      for (int t = 0; t < n_tiles; ++t) {
+        if (!warp_wait(bar_p_full + 8 * t, j & 1, abort, p.err, p.wait_limit)) { ok = false; break; }
+        if (p.debug_skip_last_pv && !more) { ok = false; break; }   // the softmax's final wait must expire
+        if (lane0) {
           tc_fence_after();
           issue_pv(t, v_tile_of(u), j > 0);
           if (more) issue_qk(t, k_tile_of(u));
           umma_commit(bar_s_full + 8 * t);   // S_t(j+1) ready -- or, after the last tile, O_t final
         }
-        if (!ok) break;
-        umma_commit(bar_empty + 8 * (u & 1));
+        __syncwarp();
       }
+      if (!ok) break;
+      if (lane0) umma_commit(bar_empty + 8 * (u & 1));
+      __syncwarp();
     }
-    __syncwarp();
   } else {
     // ------------------------------------------------------------ softmax
-    const int t = warp >> 3;                                      // 0 = tile A, 1 = tile B
-    const int c = (warp >> 2) & 1;                                // key half: columns [64c, 64c + 64)
+    const int sw = warp - kWarpSoftmax0;
+    const int t = sw >> 3;                                        // 0 = tile A, 1 = tile B
+    const int c = (sw >> 2) & 1;                                  // key half: columns [64c, 64c + 64)
     if (t == 0 || has_b) {
-      const int r = threadIdx.x & 127;                            // query row in the tile
+      const int r = (warp & 3) * 32 + (threadIdx.x & 31);         // query row in the tile = TMEM lane
       const uint32_t t_lane = tmem + (static_cast<uint32_t>((warp & 3) * 32) << 16);
       const uint32_t colS = col_s(t), colO = col_o(t);
       const uint32_t bar_s = bar_s_full + 8 * t;
@@ -336,15 +330,16 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
       const float sl2 = p.scale_log2;
       float m_used = -INFINITY;                                  // running max in use (log2 units)
       float2 l2 = make_float2(0.f, 0.f);                         // this half's row sum, two lanes
-      // O *= a over this group's half of the O columns
+      // O *= a over this group's half of the O columns (16 at a time: the
+      // tile's 64 scores stay in registers meanwhile)
       auto rescale_o = [&](float a) {
+#pragma unroll 1
+        for (int c0 = 0; c0 < D / 2; c0 += 16) {
+          uint32_t o[16];
+          tmem_ld_16(t_lane + colO + c * (D / 2) + c0, o);
 #pragma unroll
-        for (int c0 = 0; c0 < D / 2; c0 += 32) {
-          uint32_t o[32];
-          tmem_ld_32(t_lane + colO + c * (D / 2) + c0, o);
-#pragma unroll
-          for (int k = 0; k < 32; ++k) o[k] = __float_as_uint(__uint_as_float(o[k]) * a);
-          tmem_st_32(t_lane + colO + c * (D / 2) + c0, o);
+          for (int k = 0; k < 16; ++k) o[k] = __float_as_uint(__uint_as_float(o[k]) * a);
+          tmem_st_16(t_lane + colO + c * (D / 2) + c0, o);
         }
       };
       // An expired wait sets the abort flag; the groups then run on over stale
@@ -353,12 +348,10 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
         warp_wait(bar_s, j & 1, abort, p.err, p.wait_limit);
         tc_fence_after();
         const int valid = j < n_p ? min(kBN, p.P - j * kBN) : min(kBN, p.G - (j - n_p) * kBN);
-        float hm;
-        {
-          float x[64];
-          load_scores64(t_lane + colS + 64 * c, 64 * c, valid, x);
-          hm = max64(x);
-        }
+        // The group's 64 scores are read from TMEM once and kept in registers.
+        float x[64];
+        load_scores64(t_lane + colS + 64 * c, 64 * c, valid, x);
+        const float hm = max64(x);
         // A slot of parity j & 1 is rewritten at tile j + 2 only after both
         // groups passed tile j + 1's barrier, i.e. after it was read.
         slot(j & 1, c)[r] = hm * sl2;
@@ -382,19 +375,15 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
         uint32_t pk[2][16];
 #pragma unroll
         for (int q32 = 0; q32 < 2; ++q32) {
-          float x[32];
-          load_scores32(t_lane + colS + 64 * c + 32 * q32, 64 * c + 32 * q32, valid, x);
 #pragma unroll
           for (int k = 0; k < 16; ++k) {
-            const float2 y = ffma2(make_float2(x[2 * k], x[2 * k + 1]), slv, neg_m);
-            const float p0 = ex2_approx(y.x);
-            const float p1 = ex2_approx(y.y);
-            acc[k & 1] = fadd2(acc[k & 1], make_float2(p0, p1));
-            pk[q32][k] = pack_bf16x2(p0, p1);
+            const float2 y = ffma2(make_float2(x[32 * q32 + 2 * k], x[32 * q32 + 2 * k + 1]), slv, neg_m);
+            const float2 pr = make_float2(ex2_approx(y.x), ex2_approx(y.y));
+            acc[k & 1] = fadd2(acc[k & 1], pr);
+            pk[q32][k] = pack_bf16x2(pr.x, pr.y);
           }
-          // P over this group's own S columns, already read (the second
-          // chunk's S columns [32, 64) stay unwritten until read).  The store
-          // stays in flight while the next chunk is computed.
+          // P over the first 32 of this group's own S columns (all 64 already
+          // read); the store stays in flight while the next chunk is computed.
           tmem_st_16_async(t_lane + colS + 64 * c + 16 * q32, pk[q32]);
         }
         tmem_wait_st();
