@@ -180,6 +180,78 @@ int archer_should_refresh(int batch, int resp_len, const int32_t* g_cur, int32_t
 int archer_cache_rewrite(const archer_shape* shape, const void* k_src, const void* v_src,
                          void* k_dst, void* v_dst, const uint8_t* refresh_flags, void* stream);
 
+/*
+ * One denoising step of Algorithm 1 over an L-layer stack, captured once as a
+ * CUDA graph and replayed with no host synchronisation (the refresh decision
+ * stays on the device):
+ *   1. the refresh rule (archer_should_refresh with update_anchor = 1);
+ *   2. a one-CTA kernel reduces the flags and sets the graph's conditional
+ *      value to "any sequence flagged" (and adds 1 to *refresh_count if so);
+ *   3. an if/else conditional node: if any flag, every layer runs
+ *      archer_prompt_refresh with the per-sequence flags (unflagged sequences
+ *      take the cached step in the same launch; flagged ones get their cache
+ *      rewritten), else every layer runs archer_attn_step;
+ *   4. archer_decode_scores over the step's logits (skipped if logits NULL).
+ * Every pointer below is captured into the graph: the buffers must stay
+ * allocated and in place for the graph's lifetime, and each step's inputs
+ * (token ids, Q/K/V rows, logits) are written into them before the launch.
+ * One graph serves one stream at a time; launches on one stream serialise.
+ */
+typedef struct archer_layer_io {
+  const void* q_all;          /* [B, N, Hq, D]  read by a refresh            */
+  const void* q_resp;         /* [B, G, Hq, D]  read by a cached step        */
+  const void* k_prompt_new;   /* [B, P, Hkv, D] fresh prompt K (refresh)      */
+  const void* v_prompt_new;
+  const void* k_resp;         /* [B, G, Hkv, D]                              */
+  const void* v_resp;
+  void* k_cache;              /* [B, P, Hkv, D] the prompt cache C_p          */
+  void* v_cache;
+  void* out_full;             /* [B, N, Hq, D]  written by a refresh          */
+  void* out_step;             /* [B, G, Hq, D]  written by a cached step      */
+} archer_layer_io;
+
+typedef struct archer_step_desc {
+  archer_shape shape;         /* the layers' common shape                     */
+  int n_layers;               /* L >= 1                                       */
+  const archer_layer_io* layers;   /* [L], copied at creation                 */
+  /* refresh rule (see archer_should_refresh) */
+  const int32_t* g_cur;       /* [B, G] */
+  int32_t* g_anchor;          /* [B, G] */
+  int32_t* age;               /* [B]    */
+  int K;
+  int max_age;
+  int32_t* dist_out;          /* [B], may be NULL */
+  uint8_t* flag_out;          /* [B]    */
+  int32_t* refresh_count;     /* one int32, may be NULL: +1 per refreshing step */
+  /* decoder scoring (see archer_decode_scores); logits NULL skips it */
+  int vocab;
+  int logits_dtype;
+  const void* logits;         /* [B * G, row_stride] */
+  int64_t row_stride;
+  const uint8_t* mask_state;
+  const int32_t* cur_tokens;
+  float* max_prob;
+  int32_t* top1;
+  float* margin;
+  float* cur_prob;
+  void* scores_workspace;
+  size_t scores_workspace_bytes;
+} archer_step_desc;
+
+typedef struct archer_step_graph archer_step_graph;
+
+/* Validates desc, captures and instantiates the graph (host work, done once;
+ * the capture runs on a private stream and launches nothing).  *out receives
+ * the handle.  Calls no cudaMalloc; the graph's own objects are the CUDA
+ * runtime's. */
+int archer_step_graph_create(const archer_step_desc* desc, archer_step_graph** out);
+
+/* Launches one step on `stream`. */
+int archer_step_graph_launch(archer_step_graph* graph, void* stream);
+
+/* Frees the graph (after its last launch has completed). */
+int archer_step_graph_destroy(archer_step_graph* graph);
+
 /* Reads and clears the device-side error word that kernels set when a
  * bounded wait expires.  Synchronises `stream`.  Returns ARCHER_OK or
  * ARCHER_ERR_TIMEOUT (or ARCHER_ERR_CUDA). */

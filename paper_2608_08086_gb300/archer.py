@@ -40,6 +40,23 @@ class archer_shape(ctypes.Structure):
                 ("softmax_scale", ctypes.c_float)]
 
 
+class archer_layer_io(ctypes.Structure):
+    _fields_ = [(n, ctypes.c_void_p) for n in ("q_all", "q_resp", "k_prompt_new", "v_prompt_new", "k_resp",
+                                               "v_resp", "k_cache", "v_cache", "out_full", "out_step")]
+
+
+class archer_step_desc(ctypes.Structure):
+    _fields_ = [("shape", archer_shape), ("n_layers", ctypes.c_int), ("layers", ctypes.POINTER(archer_layer_io)),
+                ("g_cur", ctypes.c_void_p), ("g_anchor", ctypes.c_void_p), ("age", ctypes.c_void_p),
+                ("K", ctypes.c_int), ("max_age", ctypes.c_int), ("dist_out", ctypes.c_void_p),
+                ("flag_out", ctypes.c_void_p), ("refresh_count", ctypes.c_void_p),
+                ("vocab", ctypes.c_int), ("logits_dtype", ctypes.c_int), ("logits", ctypes.c_void_p),
+                ("row_stride", ctypes.c_int64), ("mask_state", ctypes.c_void_p), ("cur_tokens", ctypes.c_void_p),
+                ("max_prob", ctypes.c_void_p), ("top1", ctypes.c_void_p), ("margin", ctypes.c_void_p),
+                ("cur_prob", ctypes.c_void_p), ("scores_workspace", ctypes.c_void_p),
+                ("scores_workspace_bytes", ctypes.c_size_t)]
+
+
 def _load():
     if not os.path.exists(LIB_PATH):
         raise ImportError(f"{LIB_PATH} is missing: build it with paper_2608_08086_gb300.build.build() "
@@ -62,8 +79,12 @@ def _load():
     L.archer_last_error.argtypes = []
     L.archer_last_error.restype = ctypes.c_char_p
     L.archer_version.argtypes = []
+    L.archer_step_graph_create.argtypes = [ctypes.POINTER(archer_step_desc), ctypes.POINTER(vp)]
+    L.archer_step_graph_launch.argtypes = [vp, vp]
+    L.archer_step_graph_destroy.argtypes = [vp]
     for name in ("archer_attn_step", "archer_prompt_refresh", "archer_decode_scores", "archer_should_refresh",
-                 "archer_cache_rewrite", "archer_check_device", "archer_version"):
+                 "archer_cache_rewrite", "archer_check_device", "archer_version", "archer_step_graph_create",
+                 "archer_step_graph_launch", "archer_step_graph_destroy"):
         getattr(L, name).restype = ctypes.c_int
     return L
 
@@ -253,3 +274,72 @@ def archer_version() -> int:
 
 def default_scale(head_dim: int) -> float:
     return 1.0 / math.sqrt(head_dim)
+
+
+class StepGraph:
+    """One denoising step of Algorithm 1 over an L-layer stack as a CUDA graph
+    (archer_step_graph_create): rule, device-side refresh branch, L attention
+    layers, scoring.  Every tensor given here is captured by address: keep
+    them alive and write each step's inputs into them in place."""
+
+    def __init__(self, shape: archer_shape, layers, g_cur, g_anchor, age, K, max_age, flag_out, dist_out=None,
+                 refresh_count=None, logits=None, max_prob=None, top1=None, margin=None, vocab=None,
+                 mask_state=None, cur_tokens=None, cur_prob=None, workspace=None):
+        bf = torch.bfloat16
+        B, G = g_cur.shape
+        if B != shape.batch or G != shape.resp_len:
+            raise ValueError("g_cur must be [batch, resp_len]")
+        self._keep = []            # tensors whose addresses the graph holds
+        ios = (archer_layer_io * len(layers))()
+        for i, l in enumerate(layers):
+            for name in archer_layer_io._fields_:
+                t = l[name[0]]
+                self._keep.append(t)
+                setattr(ios[i], name[0], _ptr(t, bf, name[0]))
+        d = archer_step_desc()
+        d.shape = shape
+        d.n_layers = len(layers)
+        d.layers = ios
+        i32 = torch.int32
+        d.g_cur, d.g_anchor, d.age = _ptr(g_cur, i32, "g_cur"), _ptr(g_anchor, i32, "g_anchor"), _ptr(age, i32, "age")
+        d.K, d.max_age = int(min(K, K_INFINITE)), int(max_age)
+        d.dist_out = _ptr(dist_out, i32, "dist_out")
+        d.flag_out = _ptr(flag_out, torch.uint8, "flag_out")
+        d.refresh_count = _ptr(refresh_count, i32, "refresh_count")
+        self._keep += [g_cur, g_anchor, age, flag_out, dist_out, refresh_count]
+        if logits is not None:
+            if logits.dtype not in (torch.bfloat16, torch.float32):
+                raise TypeError("logits must be bf16 or fp32")
+            stride = logits.shape[-1]
+            if logits.numel() != B * G * stride:
+                raise ValueError("logits must hold batch * resp_len rows")
+            d.vocab = stride if vocab is None else int(vocab)
+            d.logits_dtype = ARCHER_DTYPE_BF16 if logits.dtype == torch.bfloat16 else ARCHER_DTYPE_F32
+            d.logits, d.row_stride = _ptr(logits, None, "logits"), stride
+            d.mask_state = _ptr(mask_state, torch.uint8, "mask_state")
+            d.cur_tokens = _ptr(cur_tokens, i32, "cur_tokens")
+            d.max_prob, d.top1 = _ptr(max_prob, torch.float32, "max_prob"), _ptr(top1, i32, "top1")
+            d.margin, d.cur_prob = _ptr(margin, torch.float32, "margin"), _ptr(cur_prob, torch.float32, "cur_prob")
+            if workspace is None:
+                workspace = scores_workspace(B * G, d.vocab, logits.device)
+            d.scores_workspace = _ptr(workspace, None, "workspace")
+            d.scores_workspace_bytes = 0 if workspace is None else workspace.numel() * workspace.element_size()
+            self._keep += [logits, mask_state, cur_tokens, max_prob, top1, margin, cur_prob, workspace]
+        h = ctypes.c_void_p()
+        _raise(lib.archer_step_graph_create(ctypes.byref(d), ctypes.byref(h)))
+        self._h = h
+
+    def launch(self, stream=None):
+        _raise(lib.archer_step_graph_launch(self._h, _stream(stream)))
+
+    def close(self):
+        if getattr(self, "_h", None):
+            torch.cuda.synchronize()
+            lib.archer_step_graph_destroy(self._h)
+            self._h = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass

@@ -13,6 +13,10 @@ in every layer each step).  Per step t:
   5. archer_decode_scores over the step's logits.
 Step 0 is the FullForward that builds every layer's prompt cache.
 ``mode="eager"`` refreshes every step (K = 0), the full-recomputation comparator.
+``mode="graph"`` runs the same rule as "archer" but each step after the build is
+one replay of an archer_step_graph (rule, device-side refresh branch, layers,
+scoring): the host never reads the flags to decide, so steps queue back to
+back.
 
 Per-layer buffers are slices of stacked tensors so that one indexed copy
 stages a redraw for all layers.  With ``source="host"`` every input comes
@@ -46,6 +50,8 @@ class DeviceTrajectory:
         self.Hq, self.Hkv, self.D = sh.n_heads, sh.n_kv_heads, sh.head_dim
         self.N = self.P + self.G
         self.L = wl.layers if layers is None else layers
+        if mode not in ("archer", "eager", "graph"):
+            raise ValueError(f"unknown mode {mode}")
         self.K = 0 if mode == "eager" else wl.radius_k
         self.max_age = 0 if mode == "eager" else wl.max_age
         self.score = score and wl.logits_rows > 0
@@ -53,7 +59,8 @@ class DeviceTrajectory:
         self.shape = A.make_shape(self.B, self.P, self.G, self.Hq, self.Hkv, self.D)
         self.pool_steps = pool_steps
         self.max_steps = wl.steps if max_steps is None else max_steps
-        self.n_refresh_steps = 0
+        self._n_refresh_steps = 0
+        self.graph = None
         self.t = -1
         self.attn_events = []          # (start, end, kind) CUDA events around attention launches
         self.time_attention = False
@@ -106,9 +113,13 @@ class DeviceTrajectory:
         self.flag_host = torch.ones(B, dtype=torch.uint8).pin_memory()
         self.out_step = torch.empty(B, G, Hq, D, dtype=bf, device=dev)
         self.out_full = torch.empty(B, N, Hq, D, dtype=bf, device=dev)
+        self.refresh_count = torch.zeros(1, dtype=torch.int32, device=dev)
         if self.score:
             rows, V = B * G, self.wl.vocab
-            if self.source == "host":
+            if self.source == "host" and self.mode == "graph":
+                dt = torch.bfloat16 if self.wl.logits_dtype == "bf16" else torch.float32
+                self.logits = torch.empty(rows, V, dtype=dt, device=dev)   # fixed: the graph holds its address
+            elif self.source == "host":
                 self.logits = None
             else:
                 dt = torch.bfloat16 if self.wl.logits_dtype == "bf16" else torch.float32
@@ -153,17 +164,22 @@ class DeviceTrajectory:
     def _score(self, t):
         if not self.score:
             return None
-        if self.source == "host":
-            z = synth.traj_logits(self.wl, self.seed, t)
-            if self.wl.logits_dtype == "bf16":
-                self.logits = _dev_bits(z, self.device)
-            else:
-                self.logits = torch.from_numpy(z).to(self.device)
+        self._upload_logits(t)
         self._timed("score", lambda: A.archer_decode_scores(self.logits, self.max_prob, self.top1, self.margin,
                                                             workspace=self.ws))
         if self.record:
             return {"max_prob": self.max_prob.clone(), "top1": self.top1.clone(), "margin": self.margin.clone()}
         return None
+
+    def _upload_logits(self, t):
+        if self.source != "host":
+            return
+        z = synth.traj_logits(self.wl, self.seed, t)
+        z = _dev_bits(z, self.device) if self.wl.logits_dtype == "bf16" else torch.from_numpy(z).to(self.device)
+        if self.mode == "graph":
+            self.logits.copy_(z)
+        else:
+            self.logits = z
 
     def _stage_redraw(self, t):
         B, P = self.B, self.P
@@ -211,12 +227,54 @@ class DeviceTrajectory:
         self.g_anchor.copy_(self.g)
         self.age.zero_()
         sc = self._score(0)
-        self.n_refresh_steps = 1
+        self._n_refresh_steps = 1
         return {"t": 0, "flag": np.ones(self.B, np.uint8), "dist": np.zeros(self.B, np.int32), "out": outs,
                 "scores": sc}
 
+    @property
+    def n_refresh_steps(self):
+        """Steps that refreshed (the build included); a device read in graph mode."""
+        if self.mode == "graph" and self.graph is not None:
+            return 1 + int(self.refresh_count.item())
+        return self._n_refresh_steps
+
+    def _make_graph(self):
+        layers = [{"q_all": self.q_all[l], "q_resp": self.q_resp[l], "k_prompt_new": self.k_new[l],
+                   "v_prompt_new": self.v_new[l], "k_resp": self.k_resp[l], "v_resp": self.v_resp[l],
+                   "k_cache": self.k_cache[l], "v_cache": self.v_cache[l], "out_full": self.out_full,
+                   "out_step": self.out_step} for l in range(self.L)]
+        sc = {}
+        if self.score:
+            sc = dict(logits=self.logits, max_prob=self.max_prob, top1=self.top1, margin=self.margin,
+                      workspace=self.ws)
+        self.refresh_count.zero_()
+        self.graph = A.StepGraph(self.shape, layers, self.g, self.g_anchor, self.age, self.K, self.max_age,
+                                 self.flag, dist_out=self.dist, refresh_count=self.refresh_count, **sc)
+
+    def _graph_step(self, t):
+        self._stage_redraw(t)
+        self._stage_fresh_prompt(t)       # host source: the graph may refresh, so the fresh prompt is staged
+        if self.score:
+            self._upload_logits(t)
+        if self.graph is None:
+            self._make_graph()
+        self.graph.launch()
+        rec = {"t": t}
+        if self.record:
+            torch.cuda.synchronize()
+            flags = self.flag.cpu().numpy()
+            refreshed = bool(flags.any())
+            # the layers share one output buffer: only the last layer's survives the replay
+            outs = [None] * (self.L - 1) + [(self.out_full if refreshed else self.out_step).clone()]
+            rec.update({"flag": flags, "out": outs, "dist": self.dist.cpu().numpy(),
+                        "scores": {"max_prob": self.max_prob.clone(), "top1": self.top1.clone(),
+                                   "margin": self.margin.clone()} if self.score else None})
+        return rec
+
     def step(self):
         t = self.t = self.t + 1
+        if self.mode == "graph":
+            return self._graph_step(t)
         self._stage_redraw(t)
         A.archer_should_refresh(self.g, self.g_anchor, self.age, self.K, self.max_age, True, self.dist, self.flag)
         self.flag_host.copy_(self.flag, non_blocking=True)
@@ -224,7 +282,7 @@ class DeviceTrajectory:
         flags = self.flag_host.numpy()
         refresh = bool(flags.any())
         if refresh:
-            self.n_refresh_steps += 1
+            self._n_refresh_steps += 1
             self._stage_fresh_prompt(t)
         outs = self._forward(refresh, self.flag if refresh else None)
         sc = self._score(t)

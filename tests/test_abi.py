@@ -82,3 +82,15 @@ def test_bad_scoring_and_rule_arguments_rejected(lib):
     assert g(-1, 4, p, p, p, 1, 0, 1, p, p, None) == -1
     assert g(2, 4, None, p, p, 1, 0, 1, p, p, None) == -1
     assert g(0, 4, None, None, None, 1, 0, 1, None, None, None) == 0
+
+
+def test_step_graph_arguments_rejected_before_any_cuda_call(lib):
+    c = lib.archer_step_graph_create
+    c.argtypes = [ctypes.c_void_p, ctypes.c_void_p]
+    out = ctypes.c_void_p(0x1234)
+    assert c(None, ctypes.byref(out)) == -1 and out.value is None      # NULL desc; *out cleared
+    assert c(None, None) == -1                                          # NULL out
+    lib.archer_step_graph_launch.argtypes = [ctypes.c_void_p, ctypes.c_void_p]
+    assert lib.archer_step_graph_launch(None, None) == -1
+    lib.archer_step_graph_destroy.argtypes = [ctypes.c_void_p]
+    assert lib.archer_step_graph_destroy(None) == 0
