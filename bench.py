@@ -549,17 +549,26 @@ def main():
     pk, pk_kind = peaks()
     clocks = ClockSampler(local)
 
-    # ---- the Archer arm (timed region = K steps)
+    # ---- the Archer arm (timed region = K steps): one step graph per step,
+    # the refresh branch taken on the device (no host synchronisation)
     clocks.start()
-    arm = run_arm(wl, "archer", args.steps, args.warmup, dist_on, time_attention=True)
+    arm = run_arm(wl, "graph", args.steps, args.warmup, dist_on)
     clk = clocks.stop()
-    tr = arm["traj"]
     ms = max_over_ranks(arm["ms"], dist_on)
     value = world * args.steps / (ms / 1e3)
+    n_ref = arm["refresh_steps"]
+    del arm
+    torch.cuda.empty_cache()
+    # ---- the same steps driven from the host (flags read back each step), with
+    # CUDA events around every attention and scoring launch: the per-kernel
+    # durations of the roofline
+    arm = run_arm(wl, "archer", args.steps, args.warmup, dist_on, time_attention=True)
+    tr = arm["traj"]
+    host_value = world * args.steps / (max_over_ranks(arm["ms"], dist_on) / 1e3)
     ks = kernel_stats(tr)
     L = tr.L
-    n_ref = arm["refresh_steps"]
-    launches = args.steps * (1 + L + (1 if tr.score else 0)) + n_ref * L   # rule + attention + scoring + rewrites
+    # per step: rule + refresh condition + L attention + scoring (2) [+ L cache rewrites on refresh steps]
+    launches = args.steps * (2 + L + (2 if tr.score else 0)) + n_ref * L
     flops_step_launch = 4.0 * tr.B * tr.Hq * tr.G * tr.N * tr.D
     flops_refresh_launch = 4.0 * tr.B * tr.Hq * tr.N * tr.N * tr.D
     att = {}
@@ -583,8 +592,8 @@ def main():
     del arm, tr
     torch.cuda.empty_cache()
 
-    # ---- the eager arm: refresh every step
-    eager = run_arm(wl, "eager", args.eager_steps, 3, dist_on)
+    # ---- the eager arm: refresh every step (one graph per step, like the Archer arm)
+    eager = run_arm(wl, "eager-graph", args.eager_steps, 3, dist_on)
     eager_ms = max_over_ranks(eager["ms"], dist_on)
     eager_value = world * args.eager_steps / (eager_ms / 1e3)
     del eager
@@ -602,17 +611,22 @@ def main():
     secondary = None
     if not args.no_secondary and args.workload != "traj32":
         wl2 = synth.WORKLOADS["traj32"]
-        a2 = run_arm(wl2, "archer", min(args.steps, 30), 3, dist_on, time_attention=True)
-        ks2 = kernel_stats(a2["traj"])
-        e2 = run_arm(wl2, "eager", args.eager_steps, 3, dist_on)
-        v2 = world * min(args.steps, 30) / (max_over_ranks(a2["ms"], dist_on) / 1e3)
+        n2 = min(args.steps, 30)
+        a2 = run_arm(wl2, "graph", n2, 3, dist_on)
+        v2 = world * n2 / (max_over_ranks(a2["ms"], dist_on) / 1e3)
+        r2 = a2["refresh_steps"]
+        del a2
+        h2 = run_arm(wl2, "archer", n2, 3, dist_on, time_attention=True)
+        ks2 = kernel_stats(h2["traj"])
+        vh2 = world * n2 / (max_over_ranks(h2["ms"], dist_on) / 1e3)
+        t2 = h2["traj"]
+        e2 = run_arm(wl2, "eager-graph", args.eager_steps, 3, dist_on)
         ve2 = world * args.eager_steps / (max_over_ranks(e2["ms"], dist_on) / 1e3)
-        t2 = a2["traj"]
         fl2 = 4.0 * t2.B * t2.Hq * t2.G * t2.N * t2.D
-        secondary = {"workload": wl2.name, "steps_per_s": v2, "eager_steps_per_s": ve2, "speedup_vs_refresh_every_step": v2 / ve2,
-                     "refresh_steps": a2["refresh_steps"],
+        secondary = {"workload": wl2.name, "steps_per_s": v2, "host_driven_steps_per_s": vh2,
+                     "eager_steps_per_s": ve2, "speedup_vs_refresh_every_step": v2 / ve2, "refresh_steps": r2,
                      "step_attention_tflops": fl2 / (ks2["step"]["mean_ms"] * 1e9) if "step" in ks2 else None}
-        del a2, e2, t2
+        del h2, e2, t2
         torch.cuda.empty_cache()
 
     # ---- CPU baseline: the oracle on a bounded sample (rank 0, N = 1)
@@ -634,6 +648,8 @@ def main():
                        "parallelism": f"replicas{world}" if world > 1 else "single",
                        "l2": "no flush: inputs larger than L2 (prompt K/V of one layer > 129 MB)"},
             "refresh_steps_timed": n_ref,
+            "step": "CUDA graph per step, refresh branch on the device",
+            "host_driven_steps_per_s": host_value,
             "speedup_vs_refresh_every_step": value / eager_value,
             "eager_steps_per_s": eager_value,
             "attention": att,

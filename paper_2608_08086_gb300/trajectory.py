@@ -13,7 +13,7 @@ in every layer each step).  Per step t:
   5. archer_decode_scores over the step's logits.
 Step 0 is the FullForward that builds every layer's prompt cache.
 ``mode="eager"`` refreshes every step (K = 0), the full-recomputation comparator.
-``mode="graph"`` runs the same rule as "archer" but each step after the build is
+``mode="graph"`` ("eager-graph") runs the same rule as "archer" ("eager") but each step after the build is
 one replay of an archer_step_graph (rule, device-side refresh branch, layers,
 scoring): the host never reads the flags to decide, so steps queue back to
 back.
@@ -50,10 +50,12 @@ class DeviceTrajectory:
         self.Hq, self.Hkv, self.D = sh.n_heads, sh.n_kv_heads, sh.head_dim
         self.N = self.P + self.G
         self.L = wl.layers if layers is None else layers
-        if mode not in ("archer", "eager", "graph"):
+        if mode not in ("archer", "eager", "graph", "eager-graph"):
             raise ValueError(f"unknown mode {mode}")
-        self.K = 0 if mode == "eager" else wl.radius_k
-        self.max_age = 0 if mode == "eager" else wl.max_age
+        self.graph_mode = mode in ("graph", "eager-graph")
+        eager = mode in ("eager", "eager-graph")
+        self.K = 0 if eager else wl.radius_k
+        self.max_age = 0 if eager else wl.max_age
         self.score = score and wl.logits_rows > 0
         self.record = record
         self.shape = A.make_shape(self.B, self.P, self.G, self.Hq, self.Hkv, self.D)
@@ -116,7 +118,7 @@ class DeviceTrajectory:
         self.refresh_count = torch.zeros(1, dtype=torch.int32, device=dev)
         if self.score:
             rows, V = B * G, self.wl.vocab
-            if self.source == "host" and self.mode == "graph":
+            if self.source == "host" and self.graph_mode:
                 dt = torch.bfloat16 if self.wl.logits_dtype == "bf16" else torch.float32
                 self.logits = torch.empty(rows, V, dtype=dt, device=dev)   # fixed: the graph holds its address
             elif self.source == "host":
@@ -176,7 +178,7 @@ class DeviceTrajectory:
             return
         z = synth.traj_logits(self.wl, self.seed, t)
         z = _dev_bits(z, self.device) if self.wl.logits_dtype == "bf16" else torch.from_numpy(z).to(self.device)
-        if self.mode == "graph":
+        if self.graph_mode:
             self.logits.copy_(z)
         else:
             self.logits = z
@@ -234,7 +236,7 @@ class DeviceTrajectory:
     @property
     def n_refresh_steps(self):
         """Steps that refreshed (the build included); a device read in graph mode."""
-        if self.mode == "graph" and self.graph is not None:
+        if self.graph_mode and self.graph is not None:
             return 1 + int(self.refresh_count.item())
         return self._n_refresh_steps
 
@@ -273,7 +275,7 @@ class DeviceTrajectory:
 
     def step(self):
         t = self.t = self.t + 1
-        if self.mode == "graph":
+        if self.graph_mode:
             return self._graph_step(t)
         self._stage_redraw(t)
         A.archer_should_refresh(self.g, self.g_anchor, self.age, self.K, self.max_age, True, self.dist, self.flag)
