@@ -63,9 +63,12 @@ typedef struct archer_shape {
  *   k_resp, v_resp [B, G, Hkv, D] bf16
  *   out     [B, G, Hq, D]  bf16 (written)
  *   lse     [B, Hq, G] fp32 (written; may be NULL)
- *   workspace / ws_bytes: scratch of at least archer_attn_workspace_size()
- *   bytes (may be NULL when that size is 0).  Owned by the caller; must not be
- *   used by another call that can overlap on the GPU.
+ *   workspace / ws_bytes: 16-byte aligned scratch of at least
+ *   archer_attn_workspace_size() bytes, any contents.  With it, a launch whose
+ *   grid leaves SMs idle splits its key tiles across CTAs and merges the
+ *   splits in a second kernel; with NULL (or too small) it runs unsplit, with
+ *   the same result up to rounding.  Owned by the caller; must not be used by
+ *   another call that can overlap on the GPU.
  * k_cache/v_cache may be NULL only when P == 0.
  */
 int archer_attn_step(const archer_shape* shape, const void* q_resp, const void* k_cache,
@@ -95,8 +98,10 @@ int archer_prompt_refresh(const archer_shape* shape, const void* q_all, const vo
                           const uint8_t* refresh_flags, void* workspace, size_t ws_bytes,
                           void* stream);
 
-/* Scratch bytes archer_attn_step / archer_prompt_refresh need for n_queries
- * (= G or N) query rows per sequence; 0 when none is needed. */
+/* Scratch bytes that let archer_attn_step / archer_prompt_refresh split the
+ * key tiles of a launch over n_queries (= G or N) query rows per sequence:
+ * n_split * B * Hq * n_queries * (4 D + 8), n_split chosen from the SM count;
+ * 0 when the launch's grid already fills the GPU (or the shape is invalid). */
 size_t archer_attn_workspace_size(const archer_shape* shape, int n_queries);
 
 /*
@@ -236,6 +241,10 @@ typedef struct archer_step_desc {
   float* cur_prob;
   void* scores_workspace;
   size_t scores_workspace_bytes;
+  /* attention scratch shared by the layers (they run one after another):
+   * archer_attn_workspace_size(shape, N) bytes let small launches split */
+  void* attn_workspace;
+  size_t attn_workspace_bytes;
 } archer_step_desc;
 
 typedef struct archer_step_graph archer_step_graph;

@@ -54,7 +54,8 @@ class archer_step_desc(ctypes.Structure):
                 ("row_stride", ctypes.c_int64), ("mask_state", ctypes.c_void_p), ("cur_tokens", ctypes.c_void_p),
                 ("max_prob", ctypes.c_void_p), ("top1", ctypes.c_void_p), ("margin", ctypes.c_void_p),
                 ("cur_prob", ctypes.c_void_p), ("scores_workspace", ctypes.c_void_p),
-                ("scores_workspace_bytes", ctypes.c_size_t)]
+                ("scores_workspace_bytes", ctypes.c_size_t), ("attn_workspace", ctypes.c_void_p),
+                ("attn_workspace_bytes", ctypes.c_size_t)]
 
 
 def _load():
@@ -128,6 +129,23 @@ def _expect(t, shape, what):
         raise ValueError(f"{what} has shape {tuple(t.shape)}, expected {tuple(shape)}")
 
 
+_attn_ws_cache: dict = {}
+
+
+def attn_workspace(shape: archer_shape, n_queries: int, device=None) -> torch.Tensor | None:
+    """A split-KV workspace for launches over n_queries rows, cached per
+    (device, size); None when the launch would not split.  Calls that may
+    overlap on the GPU must not share one."""
+    n = int(lib.archer_attn_workspace_size(ctypes.byref(shape), int(n_queries)))
+    if n == 0:
+        return None
+    dev = torch.device("cuda", torch.cuda.current_device()) if device is None else torch.device(device)
+    key = (dev, n)
+    if key not in _attn_ws_cache:
+        _attn_ws_cache[key] = torch.empty(n, dtype=torch.uint8, device=dev)
+    return _attn_ws_cache[key]
+
+
 def archer_attn_step(shape: archer_shape, q_resp, k_cache, v_cache, k_resp, v_resp, out, lse=None,
                      workspace=None, stream=None):
     """Cached response step (Sec. 4.1, Eq. archer-attention); see include/archer.h."""
@@ -143,7 +161,9 @@ def archer_attn_step(shape: archer_shape, q_resp, k_cache, v_cache, k_resp, v_re
         _expect(v_cache, (B, P, Hkv, D), "v_cache")
     if lse is not None:
         _expect(lse, (B, Hq, G), "lse")
-    ws = workspace
+    ws = attn_workspace(shape, G, q_resp.device) if workspace is None else workspace
+    if ws is False:
+        ws = None
     _raise(lib.archer_attn_step(ctypes.byref(shape), _ptr(q_resp, bf, "q_resp"), _ptr(k_cache, bf, "k_cache"),
                                 _ptr(v_cache, bf, "v_cache"), _ptr(k_resp, bf, "k_resp"), _ptr(v_resp, bf, "v_resp"),
                                 _ptr(out, bf, "out"), _ptr(lse, torch.float32, "lse"), _ptr(ws, None, "workspace"),
@@ -174,7 +194,9 @@ def archer_prompt_refresh(shape: archer_shape, q_all, k_prompt_new, v_prompt_new
         _expect(lse, (B, Hq, N), "lse")
     if refresh_flags is not None:
         _expect(refresh_flags, (B,), "refresh_flags")
-    ws = workspace
+    ws = attn_workspace(shape, N, q_all.device) if workspace is None else workspace
+    if ws is False:
+        ws = None
     _raise(lib.archer_prompt_refresh(
         ctypes.byref(shape), _ptr(q_all, bf, "q_all"), _ptr(k_prompt_new, bf, "k_prompt_new"),
         _ptr(v_prompt_new, bf, "v_prompt_new"), _ptr(k_resp, bf, "k_resp"), _ptr(v_resp, bf, "v_resp"),
@@ -325,6 +347,14 @@ class StepGraph:
             d.scores_workspace = _ptr(workspace, None, "workspace")
             d.scores_workspace_bytes = 0 if workspace is None else workspace.numel() * workspace.element_size()
             self._keep += [logits, mask_state, cur_tokens, max_prob, top1, margin, cur_prob, workspace]
+        # one scratch for every layer: the larger of the refresh and cached launches' needs
+        sizes = [int(lib.archer_attn_workspace_size(ctypes.byref(shape), m))
+                 for m in (shape.prompt_len + shape.resp_len, shape.resp_len)]
+        aws = attn_workspace(shape, (shape.prompt_len + shape.resp_len, shape.resp_len)[sizes.index(max(sizes))],
+                             g_cur.device)
+        if aws is not None:
+            d.attn_workspace, d.attn_workspace_bytes = _ptr(aws, None, "attn_workspace"), aws.numel()
+            self._keep.append(aws)
         h = ctypes.c_void_p()
         _raise(lib.archer_step_graph_create(ctypes.byref(d), ctypes.byref(h)))
         self._h = h

@@ -97,8 +97,6 @@ extern "C" {
 int archer_attn_step(const archer_shape* shape, const void* q_resp, const void* k_cache, const void* v_cache,
                      const void* k_resp, const void* v_resp, void* out, float* lse, void* workspace,
                      size_t ws_bytes, void* stream) {
-  (void)workspace;
-  (void)ws_bytes;
   float scale = 0.f;
   int st = check_shape(shape, &scale);
   if (st) return st;
@@ -116,6 +114,7 @@ int archer_attn_step(const archer_shape* shape, const void* q_resp, const void* 
   c.out = out; c.lse = lse;
   c.flags = nullptr; c.default_refresh = 0;
   c.q_begin_refresh = 0; c.q_begin_cached = 0;
+  c.ws = workspace; c.ws_bytes = ws_bytes;
   return attn_launch(c, static_cast<cudaStream_t>(stream));
 }
 
@@ -123,8 +122,6 @@ int archer_prompt_refresh(const archer_shape* shape, const void* q_all, const vo
                           const void* v_prompt_new, const void* k_resp, const void* v_resp, void* out, float* lse,
                           void* k_cache, void* v_cache, const uint8_t* refresh_flags, void* workspace,
                           size_t ws_bytes, void* stream) {
-  (void)workspace;
-  (void)ws_bytes;
   float scale = 0.f;
   int st = check_shape(shape, &scale);
   if (st) return st;
@@ -145,6 +142,7 @@ int archer_prompt_refresh(const archer_shape* shape, const void* q_all, const vo
   c.out = out; c.lse = lse;
   c.flags = refresh_flags; c.default_refresh = 1;
   c.q_begin_refresh = 0; c.q_begin_cached = c.P;
+  c.ws = workspace; c.ws_bytes = ws_bytes;
   if ((st = attn_launch(c, s))) return st;
   if (c.P == 0) return ARCHER_OK;
   const size_t per_seq = static_cast<size_t>(c.P) * c.Hkv * c.D * 2;
@@ -155,9 +153,10 @@ int archer_prompt_refresh(const archer_shape* shape, const void* q_all, const vo
 }
 
 size_t archer_attn_workspace_size(const archer_shape* shape, int n_queries) {
-  (void)shape;
-  (void)n_queries;
-  return 0;
+  float scale = 0.f;
+  if (check_shape(shape, &scale) != ARCHER_OK || n_queries < 1 || shape->batch == 0) return 0;
+  return attn_workspace_bytes(shape->batch, shape->prompt_len, shape->resp_len, shape->n_heads, shape->head_dim,
+                              n_queries);
 }
 
 int archer_cache_rewrite(const archer_shape* shape, const void* k_src, const void* v_src, void* k_dst, void* v_dst,

@@ -37,9 +37,15 @@ struct AttnCall {
   int default_refresh;    // used when flags == nullptr
   int q_begin_refresh;    // first query row of a refreshed sequence
   int q_begin_cached;     // first query row of a cached sequence
+  void* ws;               // nullable: split-KV workspace (see attn_workspace_bytes)
+  size_t ws_bytes;
 };
 
 int attn_launch(const AttnCall& c, cudaStream_t stream);
+
+// Workspace a launch over M query rows needs to split its key tiles across
+// CTAs (0 when the launch would not split: its grid already fills the GPU).
+size_t attn_workspace_bytes(int B, int P, int G, int Hq, int D, int M);
 
 int cache_rewrite_launch(int B, size_t bytes_per_seq, const void* k_src, const void* v_src,
                          void* k_dst, void* v_dst, const uint8_t* flags, cudaStream_t stream);

@@ -71,6 +71,14 @@ struct AttnParams {
   __nv_bfloat16* out;
   float* lse;
   int* err;
+  // Split over the key tiles (grids smaller than the SM count): CTA x of a
+  // launch is (query tile pair x / n_split, split x % n_split); split s takes
+  // key tiles [s * tiles_per_split, (s + 1) * tiles_per_split) of the T tiles
+  // and writes its unnormalised O, running max and row sum to the workspace
+  // instead of out; attn_combine_kernel merges the splits.
+  int n_split, tiles_per_split;
+  float* ws_o;                // [n_split, B, Hq, M, D] fp32
+  float2* ws_ml;              // [n_split, B, Hq, M] (max in log2 units, row sum)
 };
 
 template <int D>
@@ -173,7 +181,10 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
   using L = Layout<D>;
   extern __shared__ uint8_t smem_raw[];
 
-  const int tp = blockIdx.x, h = blockIdx.y, b = blockIdx.z;
+  const int tp = blockIdx.x / p.n_split, split = blockIdx.x % p.n_split, h = blockIdx.y, b = blockIdx.z;
+  // Lets a programmatic dependent (the split merge) be scheduled once every CTA
+  // of this grid is resident; it still waits for this grid's completion.
+  asm volatile("griddepcontrol.launch_dependents;");
   const bool refresh = p.flags ? (p.flags[b] != 0) : (p.default_refresh != 0);
   const int q0 = (refresh ? p.q_begin_refresh : p.q_begin_cached) + tp * 2 * kBM;
   if (q0 >= p.M) return;  // uniform over the CTA, before any barrier or TMEM use
@@ -182,7 +193,10 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
   const int kvh = h / (p.Hq / p.Hkv);
   const int n_p = (p.P + kBN - 1) / kBN;
   const int n_g = (p.G + kBN - 1) / kBN;
-  const int T = n_p + n_g;
+  const int j0 = split * p.tiles_per_split;                        // this CTA's first key tile
+  const int T = min(n_p + n_g, j0 + p.tiles_per_split) - j0;      // and its number of tiles
+  if (T <= 0) return;      // the host sizes splits so that none is empty; uniform anyway
+  const bool partial = p.n_split > 1;
 
   const uint32_t raw = smem_u32(smem_raw);
   const uint32_t base = (raw + 1023u) & ~1023u;
@@ -244,7 +258,7 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
         const bool has_v = u >= 1, has_k = u < T;
         mbar_arrive_expect_tx(bar_full + 8 * slot, (has_v && has_k ? 2 : 1) * L::kTile);
         for (int part = has_v ? 0 : 1; part < (has_k ? 2 : 1); ++part) {
-          const int j = part == 0 ? u - 1 : u;
+          const int j = j0 + (part == 0 ? u - 1 : u);             // global key tile
           const bool in_prompt = j < n_p;
           const int row = in_prompt ? j * kBN : (j - n_p) * kBN;
           const CUtensorMap* map = in_prompt ? (part == 0 ? mVp : mKp) : (part == 0 ? &tmVg : &tmKg);
@@ -347,7 +361,8 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
       for (int j = 0; j < T; ++j) {
         warp_wait(bar_s, j & 1, abort, p.err, p.wait_limit);
         tc_fence_after();
-        const int valid = j < n_p ? min(kBN, p.P - j * kBN) : min(kBN, p.G - (j - n_p) * kBN);
+        const int jg = j0 + j;                                    // global key tile
+        const int valid = jg < n_p ? min(kBN, p.P - jg * kBN) : min(kBN, p.G - (jg - n_p) * kBN);
         // The group's 64 scores are read from TMEM once and kept in registers.
         float x[64];
         load_scores64(t_lane + colS + 64 * c, 64 * c, valid, x);
@@ -398,26 +413,45 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
       slot(0, c)[r] = l2.x + l2.y;
       tile_bar(t);
       const float l_sum = slot(0, c)[r] + slot(0, c ^ 1)[r];
-      const float inv_l = 1.0f / l_sum;
       const int q = q0 + t * kBM + r;
       const bool live = ok && q < p.M;
-      __nv_bfloat16* orow = p.out + ((static_cast<size_t>(b) * p.M + q) * p.Hq + h) * D + c * (D / 2);
+      if (partial) {
+        // unnormalised O, max and sum of this key range, merged by the combine kernel
+        const size_t row = ((static_cast<size_t>(split) * gridDim.z + b) * p.Hq + h) * p.M + q;
+        float* orow_ws = p.ws_o + row * D + c * (D / 2);
 #pragma unroll
-      for (int c0 = 0; c0 < D / 2; c0 += 32) {
-        uint32_t o[32];
-        tmem_ld_32(t_lane + colO + c * (D / 2) + c0, o);
-        uint32_t w[16];
+        for (int c0 = 0; c0 < D / 2; c0 += 32) {
+          uint32_t o[32];
+          tmem_ld_32(t_lane + colO + c * (D / 2) + c0, o);
+          if (live) {
+            float4* dst = reinterpret_cast<float4*>(orow_ws + c0);
 #pragma unroll
-        for (int k = 0; k < 16; ++k)
-          w[k] = pack_bf16x2(__uint_as_float(o[2 * k]) * inv_l, __uint_as_float(o[2 * k + 1]) * inv_l);
-        if (live) {
-          uint4* dst = reinterpret_cast<uint4*>(orow + c0);
-#pragma unroll
-          for (int v = 0; v < 4; ++v) dst[v] = make_uint4(w[4 * v], w[4 * v + 1], w[4 * v + 2], w[4 * v + 3]);
+            for (int v = 0; v < 8; ++v)
+              dst[v] = make_float4(__uint_as_float(o[4 * v]), __uint_as_float(o[4 * v + 1]),
+                                   __uint_as_float(o[4 * v + 2]), __uint_as_float(o[4 * v + 3]));
+          }
         }
+        if (live && c == 0) p.ws_ml[row] = make_float2(m_used, l_sum);
+      } else {
+        const float inv_l = 1.0f / l_sum;
+        __nv_bfloat16* orow = p.out + ((static_cast<size_t>(b) * p.M + q) * p.Hq + h) * D + c * (D / 2);
+#pragma unroll
+        for (int c0 = 0; c0 < D / 2; c0 += 32) {
+          uint32_t o[32];
+          tmem_ld_32(t_lane + colO + c * (D / 2) + c0, o);
+          uint32_t w[16];
+#pragma unroll
+          for (int k = 0; k < 16; ++k)
+            w[k] = pack_bf16x2(__uint_as_float(o[2 * k]) * inv_l, __uint_as_float(o[2 * k + 1]) * inv_l);
+          if (live) {
+            uint4* dst = reinterpret_cast<uint4*>(orow + c0);
+#pragma unroll
+            for (int v = 0; v < 4; ++v) dst[v] = make_uint4(w[4 * v], w[4 * v + 1], w[4 * v + 2], w[4 * v + 3]);
+          }
+        }
+        if (live && c == 0 && p.lse)
+          p.lse[(static_cast<size_t>(b) * p.Hq + h) * p.M + q] = (m_used + log2f(l_sum)) * 0.69314718055994531f;
       }
-      if (live && c == 0 && p.lse)
-        p.lse[(static_cast<size_t>(b) * p.Hq + h) * p.M + q] = (m_used + log2f(l_sum)) * 0.69314718055994531f;
     }
   }
 
@@ -430,7 +464,90 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
   }
 }
 
+// Merges the key-range splits of one output row (b, q, h): with m_s the
+// split's running max (log2 units), l_s its row sum and O_s its unnormalised
+// output, out = sum_s 2^(m_s - m) O_s / sum_s 2^(m_s - m) l_s, m = max_s m_s.
+// One thread per 8 output columns of a row; rows a launch did not compute
+// (below q_begin) are left alone.  Launched as a programmatic dependent of the
+// attention kernel: it waits for that grid before reading the workspace.
+template <int D>
+__global__ void __launch_bounds__(256)
+attn_combine_kernel(const float* __restrict__ ws_o, const float2* __restrict__ ws_ml, int n_split, int B, int Hq,
+                    int M, const uint8_t* __restrict__ flags, int default_refresh, int q_begin_refresh,
+                    int q_begin_cached, __nv_bfloat16* __restrict__ out, float* __restrict__ lse) {
+  constexpr int kChunks = D / 8;
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+  const long long idx = static_cast<long long>(blockIdx.x) * blockDim.x + threadIdx.x;
+  const long long rows = static_cast<long long>(B) * M * Hq;
+  if (idx >= rows * kChunks) return;
+  const int ch = static_cast<int>(idx % kChunks);
+  const long long r = idx / kChunks;                              // [b][q][h] order, as out
+  const int h = static_cast<int>(r % Hq);
+  const int q = static_cast<int>((r / Hq) % M);
+  const int b = static_cast<int>(r / (static_cast<long long>(Hq) * M));
+  const bool refresh = flags ? (flags[b] != 0) : (default_refresh != 0);
+  if (q < (refresh ? q_begin_refresh : q_begin_cached)) return;
+  const size_t row0 = (static_cast<size_t>(b) * Hq + h) * M + q;   // workspace [split][b][h][q]
+  const size_t stride = static_cast<size_t>(B) * Hq * M;
+  float m = -INFINITY;
+  for (int sp = 0; sp < n_split; ++sp) m = fmaxf(m, ws_ml[sp * stride + row0].x);
+  float acc[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+  float l = 0.f;
+#pragma unroll 4
+  for (int sp = 0; sp < n_split; ++sp) {
+    const float2 ml = ws_ml[sp * stride + row0];
+    const float w = ex2_approx(ml.x - m);
+    l += w * ml.y;
+    const float4* o = reinterpret_cast<const float4*>(ws_o + (sp * stride + row0) * D + ch * 8);
+    const float4 a0 = o[0], a1 = o[1];
+    acc[0] += w * a0.x; acc[1] += w * a0.y; acc[2] += w * a0.z; acc[3] += w * a0.w;
+    acc[4] += w * a1.x; acc[5] += w * a1.y; acc[6] += w * a1.z; acc[7] += w * a1.w;
+  }
+  const float inv_l = 1.0f / l;
+  *reinterpret_cast<uint4*>(out + ((static_cast<size_t>(b) * M + q) * Hq + h) * D + ch * 8) =
+      make_uint4(pack_bf16x2(acc[0] * inv_l, acc[1] * inv_l), pack_bf16x2(acc[2] * inv_l, acc[3] * inv_l),
+                 pack_bf16x2(acc[4] * inv_l, acc[5] * inv_l), pack_bf16x2(acc[6] * inv_l, acc[7] * inv_l));
+  if (lse && ch == 0) lse[(static_cast<size_t>(b) * Hq + h) * M + q] = (m + log2f(l)) * 0.69314718055994531f;
+}
+
 // ------------------------------------------------------------------ host side
+
+constexpr int kMaxSplit = 16;
+constexpr int kMinSplitTiles = 8;   // fewer key tiles: no split
+
+int sm_count() {
+  static int count[64] = {0};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 0;
+  if (count[dev] == 0) cudaDeviceGetAttribute(&count[dev], cudaDevAttrMultiProcessorCount, dev);
+  return count[dev];
+}
+
+struct SplitPlan {
+  int n_split = 1, per = 0;
+  size_t bytes = 0;
+};
+
+// Splits the T key tiles when the grid (query tile pairs x heads x batch)
+// leaves SMs idle and the tiles are many enough to pay for the merge: as many
+// splits as whole grids fit on the SMs, none empty.  Measured on the GB300
+// (B 1, 32 heads, G 256): P 2048 (T 18) 38 -> 26 us, P 1024 (T 10) 26 -> 23 us,
+// while T <= 6 gains nothing over a CTA's fixed start-up and the merge.
+SplitPlan split_plan(int B, int P, int G, int Hq, int D, int rows, int M) {
+  SplitPlan sp;
+  const int T = (P + kBN - 1) / kBN + (G + kBN - 1) / kBN;
+  sp.per = T;
+  const long long ctas = static_cast<long long>((rows + 2 * kBM - 1) / (2 * kBM)) * Hq * B;
+  const int sms = sm_count();
+  if (ctas <= 0 || sms <= 0 || ctas >= sms || T < kMinSplitTiles) return sp;
+  int s = static_cast<int>(std::min<long long>(std::min(T, kMaxSplit), sms / ctas));
+  if (s < 2) return sp;
+  sp.per = (T + s - 1) / s;
+  sp.n_split = (T + sp.per - 1) / sp.per;
+  if (sp.n_split < 2) { sp.n_split = 1; sp.per = T; return sp; }
+  sp.bytes = static_cast<size_t>(sp.n_split) * B * Hq * M * (static_cast<size_t>(D) * 4 + 8);
+  return sp;
+}
 
 PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
   static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
@@ -503,9 +620,40 @@ int launch_d(const AttnCall& c, cudaStream_t stream) {
   prm.err = device_error_word();
   // Query tiles needed by the longest query range (a refreshed sequence's).
   const int rows = c.M - (c.flags || c.default_refresh ? c.q_begin_refresh : c.q_begin_cached);
-  const dim3 grid((rows + 2 * kBM - 1) / (2 * kBM), c.Hq, c.B);
+  SplitPlan sp = split_plan(c.B, c.P, c.G, c.Hq, D, rows, c.M);
+  if (sp.n_split > 1 && (!c.ws || c.ws_bytes < sp.bytes || (reinterpret_cast<uintptr_t>(c.ws) & 15u))) {
+    sp.n_split = 1;                                 // no (usable) workspace: one CTA per tile pair
+    sp.per = (c.P + kBN - 1) / kBN + (c.G + kBN - 1) / kBN;
+  }
+  prm.n_split = sp.n_split;
+  prm.tiles_per_split = sp.per;
+  prm.ws_o = nullptr;
+  prm.ws_ml = nullptr;
+  if (sp.n_split > 1) {
+    prm.ws_o = static_cast<float*>(c.ws);
+    prm.ws_ml = reinterpret_cast<float2*>(static_cast<char*>(c.ws) +
+                                          static_cast<size_t>(sp.n_split) * c.B * c.Hq * c.M * D * 4);
+  }
+  const dim3 grid(((rows + 2 * kBM - 1) / (2 * kBM)) * sp.n_split, c.Hq, c.B);
   attn_fwd_kernel<D><<<grid, kThreads, L::kSmemBytes, stream>>>(mq, mkr, mvr, mkc, mvc, mkg, mvg, prm);
-  return cuda_status(cudaGetLastError(), "attention launch");
+  int st = cuda_status(cudaGetLastError(), "attention launch");
+  if (st || sp.n_split == 1) return st;
+  // The merge is a programmatic dependent launch: it is scheduled while the
+  // attention grid still runs and waits for it on the device.
+  const long long threads = static_cast<long long>(c.B) * c.M * c.Hq * (D / 8);
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(static_cast<unsigned>((threads + 255) / 256));
+  cfg.blockDim = dim3(256);
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cuda_status(cudaLaunchKernelEx(&cfg, attn_combine_kernel<D>, static_cast<const float*>(prm.ws_o),
+                                        static_cast<const float2*>(prm.ws_ml), sp.n_split, c.B, c.Hq, c.M, c.flags,
+                                        c.default_refresh, c.q_begin_refresh, c.q_begin_cached, prm.out, prm.lse),
+                     "attention combine launch");
 }
 
 // Bit-exact copy of each flagged sequence's prompt K/V (16-byte words); a
@@ -524,6 +672,10 @@ __global__ void cache_rewrite_kernel(const uint4* __restrict__ k_src, const uint
 }
 
 }  // namespace
+
+size_t attn_workspace_bytes(int B, int P, int G, int Hq, int D, int M) {
+  return split_plan(B, P, G, Hq, D, M, M).bytes;
+}
 
 int attn_launch(const AttnCall& c, cudaStream_t stream) {
   if (c.B == 0) return ARCHER_OK;

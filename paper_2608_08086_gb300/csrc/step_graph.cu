@@ -66,9 +66,10 @@ int capture_layers(const archer_step_desc& d, const std::vector<archer_layer_io>
     const archer_layer_io& x = io[l];
     int st = refresh
         ? archer_prompt_refresh(&d.shape, x.q_all, x.k_prompt_new, x.v_prompt_new, x.k_resp, x.v_resp, x.out_full,
-                                nullptr, x.k_cache, x.v_cache, d.flag_out, nullptr, 0, s)
+                                nullptr, x.k_cache, x.v_cache, d.flag_out, d.attn_workspace,
+                                d.attn_workspace_bytes, s)
         : archer_attn_step(&d.shape, x.q_resp, x.k_cache, x.v_cache, x.k_resp, x.v_resp, x.out_step, nullptr,
-                           nullptr, 0, s);
+                           d.attn_workspace, d.attn_workspace_bytes, s);
     if (st) return st;
   }
   return ARCHER_OK;

@@ -63,7 +63,9 @@ ATTN_CASES = [
     (1, 300, 1, 4, 4, 64),         # G = 1
     (2, 256, 256, 2, 2, 128),      # several full tiles in both segments
     (1, 129, 130, 4, 1, 64),       # one-past-a-tile in both segments, GQA 4:1
-    (1, 640, 384, 7, 1, 128),      # GQA 7:1, 8 KV tiles
+    (1, 640, 384, 7, 1, 128),      # GQA 7:1, 8 KV tiles (split over the key tiles)
+    (1, 1500, 70, 3, 1, 64),       # 13 KV tiles, ragged tails: 13 splits of one tile
+    (2, 1500, 70, 8, 2, 64),       # 13 KV tiles over 7 splits of 2 + 2 + ... + 1 tiles
 ]
 
 
@@ -76,7 +78,8 @@ def _inputs(case, seed, std=None):
 
 @pytest.mark.parametrize("case", ATTN_CASES)
 @pytest.mark.parametrize("sharp", [False, True])
-def test_attn_step_matches_oracle(A, case, sharp):
+@pytest.mark.parametrize("split", [True, False], ids=["split", "unsplit"])
+def test_attn_step_matches_oracle(A, case, sharp, split):
     B, P, G, Hq, Hkv, D = case
     sh, bits, x = _inputs(case, seed=21, std=1.0 if sharp else None)
     scale = 1.0 if sharp else 1.0 / math.sqrt(D)
@@ -84,8 +87,12 @@ def test_attn_step_matches_oracle(A, case, sharp):
     q_resp = d["q_all"][:, P:].contiguous()
     out = torch.empty(B, G, Hq, D, dtype=torch.bfloat16, device="cuda")
     lse = torch.empty(B, Hq, G, dtype=torch.float32, device="cuda")
-    A.archer_attn_step(A.make_shape(B, P, G, Hq, Hkv, D, scale), q_resp, d["k_cache"], d["v_cache"],
-                       d["k_resp"], d["v_resp"], out, lse)
+    shape = A.make_shape(B, P, G, Hq, Hkv, D, scale)
+    if split and (P + 127) // 128 + (G + 127) // 128 >= 8:
+        # a grid that leaves SMs idle over 8+ key tiles: the tiles are split across CTAs and merged
+        assert A.archer_attn_workspace_size(shape, G) > 0
+    A.archer_attn_step(shape, q_resp, d["k_cache"], d["v_cache"], d["k_resp"], d["v_resp"], out, lse,
+                       workspace=None if split else False)
     torch.cuda.synchronize()
     A.archer_check_device()
     ref, ref_lse = O.attn_step(x["q_all"][:, P:], x["k_cache"], x["v_cache"], x["k_resp"], x["v_resp"], scale)
@@ -94,7 +101,8 @@ def test_attn_step_matches_oracle(A, case, sharp):
 
 
 @pytest.mark.parametrize("case", ATTN_CASES)
-def test_prompt_refresh_matches_oracle(A, case):
+@pytest.mark.parametrize("split", [True, False], ids=["split", "unsplit"])
+def test_prompt_refresh_matches_oracle(A, case, split):
     B, P, G, Hq, Hkv, D = case
     sh, bits, x = _inputs(case, seed=22)
     scale = 1.0 / math.sqrt(D)
@@ -104,7 +112,7 @@ def test_prompt_refresh_matches_oracle(A, case):
     lse = torch.empty(B, Hq, N, dtype=torch.float32, device="cuda")
     kc, vc = d["k_cache"].clone(), d["v_cache"].clone()
     A.archer_prompt_refresh(A.make_shape(B, P, G, Hq, Hkv, D), d["q_all"], d["k_prompt"], d["v_prompt"],
-                            d["k_resp"], d["v_resp"], out, lse, kc, vc)
+                            d["k_resp"], d["v_resp"], out, lse, kc, vc, workspace=None if split else False)
     torch.cuda.synchronize()
     A.archer_check_device()
     ref, ref_lse, rkc, rvc = O.prompt_refresh(x["q_all"], x["k_prompt"], x["v_prompt"], x["k_resp"], x["v_resp"],
@@ -150,10 +158,12 @@ def test_refresh_every_step_equals_eager_on_gpu(A):
     shape = A.make_shape(B, P, G, Hq, Hkv, D)
     out_full = torch.empty(B, N, Hq, D, dtype=torch.bfloat16, device="cuda")
     kc, vc = d["k_cache"].clone(), d["v_cache"].clone()
+    # unsplit launches (no workspace): each row's key tiles in one CTA, in the same order
     A.archer_prompt_refresh(shape, d["q_all"], d["k_prompt"], d["v_prompt"], d["k_resp"], d["v_resp"], out_full,
-                            None, kc, vc)
+                            None, kc, vc, workspace=False)
     out_step = torch.empty(B, G, Hq, D, dtype=torch.bfloat16, device="cuda")
-    A.archer_attn_step(shape, d["q_all"][:, P:].contiguous(), kc, vc, d["k_resp"], d["v_resp"], out_step)
+    A.archer_attn_step(shape, d["q_all"][:, P:].contiguous(), kc, vc, d["k_resp"], d["v_resp"], out_step,
+                       workspace=False)
     torch.cuda.synchronize()
     ref = O.attn_step(x["q_all"][:, P:], x["k_prompt"], x["v_prompt"], x["k_resp"], x["v_resp"],
                       1 / math.sqrt(D))[0]
