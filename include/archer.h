@@ -179,6 +179,24 @@ int archer_should_refresh(int batch, int resp_len, const int32_t* g_cur, int32_t
                           int32_t* age, int K, int max_age, int update_anchor, int32_t* dist_out,
                           uint8_t* flag_out, void* stream);
 
+/*
+ * Synthetic rollback decoder (a stand-in for the decoder D that Algorithm 1
+ * takes as given; the paper's method has no counterpart -- it is the
+ * environment the refresh rule reacts to).  Per sequence, from the scores of
+ * the previous step (archer_decode_scores with mask_state = (g == mask_token)
+ * and cur_tokens = g):
+ *   a masked position with max_prob >= tau_accept takes its top-1 token;
+ *   an unmasked position with cur_prob < tau_remask is masked again;
+ *   if masked positions remain and none was accepted, the masked position
+ *   with the largest max_prob (lowest index on ties) takes its top-1.
+ *   g [batch, resp_len] int32 (updated in place); max_prob, top1, cur_prob
+ *   [batch * resp_len]; changed [batch, resp_len] uint8 (written: 1 where g
+ *   changed).  Decisions in fp32.
+ */
+int archer_decoder_update(int batch, int resp_len, float tau_accept, float tau_remask,
+                          int32_t mask_token, const float* max_prob, const int32_t* top1,
+                          const float* cur_prob, int32_t* g, uint8_t* changed, void* stream);
+
 /* Bit-exact copy of a refreshed sequence's prompt K/V into the cache
  * (the cache rewrite C_r <- C_p(g_t) of Algorithm 1) for sequences whose flag
  * is set (all when flags is NULL).  src/dst [B, P, Hkv, D] bf16. */

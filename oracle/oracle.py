@@ -178,3 +178,40 @@ def should_refresh(g_cur, g_anchor, age, K, max_age, update_anchor=True):
                                        int(max_age), int(bool(update_anchor)), _ptr(dist, _ip),
                                        _ptr(flag, _up)))
     return dist, flag, ga, ag
+
+
+def decoder_update(g, max_prob, top1, cur_prob, tau_accept, tau_remask, mask_token=-1):
+    """Confidence-threshold rollback decoder, the synthetic stand-in for the
+    decoder D of Algorithm 1 (Sec. 4.2; its decisions read the scoring
+    outputs, the decoder-control inputs of Sec. 6).  Per sequence, from the
+    scores of the previous step's logits:
+      * a masked position whose max_prob >= tau_accept takes its top-1 token;
+      * an unmasked position whose current token has probability
+        cur_prob < tau_remask is masked again (rolled back);
+      * if masked positions remain and none was accepted, the masked position
+        with the largest max_prob (lowest index on ties) takes its top-1.
+    Plain loops over positions; g [B, G] int32, scores [B * G].  Returns
+    (g', changed [B, G] uint8)."""
+    g = np.array(g, dtype=np.int32, copy=True)
+    B, G = g.shape
+    mp = np.asarray(max_prob, dtype=np.float64).reshape(B, G)
+    t1 = np.asarray(top1, dtype=np.int64).reshape(B, G)
+    cp = np.asarray(cur_prob, dtype=np.float64).reshape(B, G)
+    changed = np.zeros((B, G), dtype=np.uint8)
+    for b in range(B):
+        accepted = False
+        best, best_i = -1.0, -1
+        old = g[b].copy()
+        for i in range(G):
+            if old[i] == mask_token:
+                if mp[b, i] > best:
+                    best, best_i = mp[b, i], i
+                if mp[b, i] >= tau_accept:
+                    g[b, i] = t1[b, i]
+                    accepted = True
+            elif cp[b, i] < tau_remask:
+                g[b, i] = mask_token
+        if not accepted and best_i >= 0:
+            g[b, best_i] = t1[b, best_i]
+        changed[b] = (g[b] != old).astype(np.uint8)
+    return g, changed

@@ -13,6 +13,11 @@ algorithm's order:
            else:    CachedForward per layer (response queries over [cache || response])
            score the step's logits.
 ``mode="eager"`` forces a refresh every step (K = 0, Eq. archer-fresh).
+``decoder="closed"`` replaces the redraw by a confidence rule on the previous
+step's scores (oracle.decoder_update): every position starts masked, a
+changed position gets new Q/K/V rows (synth.closed_loop_rows), and the logits
+plant a target token per position whose boost grows with the step
+(synth.closed_loop_logits), so refresh decisions depend on scoring outputs.
 """
 from __future__ import annotations
 
@@ -29,7 +34,7 @@ def _f64(bits):
 
 
 def run(wl: synth.Workload, seed: int = 0, mode: str = "archer", steps: int | None = None,
-        n_threads: int = 0, score: bool = True) -> list:
+        n_threads: int = 0, score: bool = True, decoder: str = "redraw", closed_loop: dict | None = None) -> list:
     sh = wl.shape
     B, P, G, Hq, Hkv, D = sh.batch, sh.prompt_len, sh.resp_len, sh.n_heads, sh.n_kv_heads, sh.head_dim
     N = P + G
@@ -38,13 +43,23 @@ def run(wl: synth.Workload, seed: int = 0, mode: str = "archer", steps: int | No
     scale = 1.0 / math.sqrt(D)
     T = wl.steps if steps is None else steps
 
-    g = synth.traj_initial_tokens(wl, seed)
+    closed = decoder == "closed"
+    cl = dict(synth.CLOSED_LOOP, **(closed_loop or {}))
+    if closed:
+        g = np.full((B, G), synth.MASK_TOKEN, dtype=np.int32)
+    else:
+        g = synth.traj_initial_tokens(wl, seed)
     layers = []
     for layer in range(wl.layers):
         x = synth.traj_layer_initial(wl, seed, layer)
         layers.append({k: _f64(v) for k, v in x.items()})
 
     def scores(t):
+        if closed:
+            z = synth.closed_loop_logits(wl, seed, t, cl["boost_per_step"])
+            z = _f64(z) if wl.logits_dtype == "bf16" else z.astype(np.float64)
+            return O.decode_scores(z, mask_state=(g == synth.MASK_TOKEN).astype(np.uint8), cur_tokens=g,
+                                   n_threads=n_threads)
         if not score or wl.logits_rows == 0:
             return None
         z = synth.traj_logits(wl, seed, t)
@@ -60,19 +75,32 @@ def run(wl: synth.Workload, seed: int = 0, mode: str = "archer", steps: int | No
         x["k_cache"], x["v_cache"] = kc, vc
         rec["out"].append(out)
     rec["scores"] = scores(0)
+    rec["g"] = g.copy()
     records = [rec]
     g_anchor = g.copy()
     age = np.zeros(B, np.int32)
 
     for t in range(1, T + 1):
-        pos, new = synth.traj_redraw(wl, seed, t, g)
-        bidx = np.arange(B)[:, None]
-        g[bidx, pos] = new
-        for layer, x in enumerate(layers):
-            rows = synth.traj_redraw_rows(wl, seed, t, layer)
-            x["q_all"][bidx, P + pos] = _f64(rows["q"])
-            x["k_resp"][bidx, pos] = _f64(rows["k"])
-            x["v_resp"][bidx, pos] = _f64(rows["v"])
+        changed = None
+        if closed:
+            prev = records[-1]["scores"]
+            g, changed = O.decoder_update(g, prev["max_prob"], prev["top1"], prev["cur_prob"],
+                                          cl["tau_accept"], cl["tau_remask"], synth.MASK_TOKEN)
+            bs, ps = np.nonzero(changed)
+            for layer, x in enumerate(layers):
+                rows = synth.closed_loop_rows(wl, seed, t, layer)
+                x["q_all"][bs, P + ps] = _f64(rows["q"][bs, ps])
+                x["k_resp"][bs, ps] = _f64(rows["k"][bs, ps])
+                x["v_resp"][bs, ps] = _f64(rows["v"][bs, ps])
+        else:
+            pos, new = synth.traj_redraw(wl, seed, t, g)
+            bidx = np.arange(B)[:, None]
+            g[bidx, pos] = new
+            for layer, x in enumerate(layers):
+                rows = synth.traj_redraw_rows(wl, seed, t, layer)
+                x["q_all"][bidx, P + pos] = _f64(rows["q"])
+                x["k_resp"][bidx, pos] = _f64(rows["k"])
+                x["v_resp"][bidx, pos] = _f64(rows["v"])
         dist, flag, g_anchor, age = O.should_refresh(g, g_anchor, age, K, max_age, update_anchor=True)
         rec = {"t": t, "flag": flag, "dist": dist, "out": []}
         if flag.any():
@@ -91,5 +119,7 @@ def run(wl: synth.Workload, seed: int = 0, mode: str = "archer", steps: int | No
                                        scale, n_threads=n_threads)
                 rec["out"].append(out)
         rec["scores"] = scores(t)
+        rec["g"] = g.copy()
+        rec["changed"] = changed
         records.append(rec)
     return records

@@ -74,6 +74,8 @@ def _load():
     L.archer_decode_scores_workspace_size.restype = sz
     L.archer_should_refresh.argtypes = [i, i, vp, vp, vp, i, i, i, vp, vp, vp]
     L.archer_cache_rewrite.argtypes = [sp, vp, vp, vp, vp, vp, vp]
+    L.archer_decoder_update.argtypes = [i, i, ctypes.c_float, ctypes.c_float, ctypes.c_int32, vp, vp, vp, vp, vp,
+                                        vp]
     L.archer_check_device.argtypes = [vp]
     L.archer_status_string.argtypes = [i]
     L.archer_status_string.restype = ctypes.c_char_p
@@ -85,6 +87,7 @@ def _load():
     L.archer_step_graph_destroy.argtypes = [vp]
     for name in ("archer_attn_step", "archer_prompt_refresh", "archer_decode_scores", "archer_should_refresh",
                  "archer_cache_rewrite", "archer_check_device", "archer_version", "archer_step_graph_create",
+                 "archer_decoder_update",
                  "archer_step_graph_launch", "archer_step_graph_destroy"):
         getattr(L, name).restype = ctypes.c_int
     return L
@@ -277,6 +280,21 @@ def archer_should_refresh(g_cur, g_anchor, age, K, max_age, update_anchor, dist_
                                      _ptr(age, i32, "age"), int(min(K, K_INFINITE)), int(max_age),
                                      int(bool(update_anchor)), _ptr(dist_out, i32, "dist_out"),
                                      _ptr(flag_out, torch.uint8, "flag_out"), _stream(stream)))
+
+
+def archer_decoder_update(g, max_prob, top1, cur_prob, changed, tau_accept, tau_remask, mask_token=-1,
+                          stream=None):
+    """Synthetic rollback decoder (stand-in for D); see include/archer.h."""
+    B, G = g.shape
+    _expect(changed, (B, G), "changed")
+    for t, n, dt in ((max_prob, "max_prob", torch.float32), (top1, "top1", torch.int32),
+                     (cur_prob, "cur_prob", torch.float32)):
+        if t.numel() != B * G or t.dtype != dt:
+            raise ValueError(f"{n} must hold {B * G} {dt} values")
+    _raise(lib.archer_decoder_update(B, G, float(tau_accept), float(tau_remask), int(mask_token),
+                                     _ptr(max_prob, None, "max_prob"), _ptr(top1, None, "top1"),
+                                     _ptr(cur_prob, None, "cur_prob"), _ptr(g, torch.int32, "g"),
+                                     _ptr(changed, torch.uint8, "changed"), _stream(stream)))
 
 
 def archer_cache_rewrite(shape: archer_shape, k_src, v_src, k_dst, v_dst, refresh_flags=None, stream=None):

@@ -211,6 +211,20 @@ int archer_should_refresh(int batch, int resp_len, const int32_t* g_cur, int32_t
                                static_cast<cudaStream_t>(stream));
 }
 
+int archer_decoder_update(int batch, int resp_len, float tau_accept, float tau_remask, int32_t mask_token,
+                          const float* max_prob, const int32_t* top1, const float* cur_prob, int32_t* g,
+                          uint8_t* changed, void* stream) {
+  if (batch < 0 || resp_len < 0) { set_error("bad shape: batch=%d resp_len=%d", batch, resp_len); return ARCHER_ERR_ARG; }
+  if (batch == 0 || resp_len == 0) return ARCHER_OK;
+  if (!max_prob || !top1 || !cur_prob || !g || !changed) {
+    set_error("max_prob, top1, cur_prob, g and changed must not be NULL");
+    return ARCHER_ERR_ARG;
+  }
+  if (!(tau_accept == tau_accept) || !(tau_remask == tau_remask)) { set_error("thresholds must not be NaN"); return ARCHER_ERR_ARG; }
+  return decoder_update_launch(batch, resp_len, tau_accept, tau_remask, mask_token, max_prob, top1, cur_prob, g,
+                               changed, static_cast<cudaStream_t>(stream));
+}
+
 int archer_check_device(void* stream) {
   cudaError_t e = cudaStreamSynchronize(static_cast<cudaStream_t>(stream));
   if (e != cudaSuccess) return cuda_status(e, "cudaStreamSynchronize");

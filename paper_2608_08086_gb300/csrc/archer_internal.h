@@ -56,6 +56,10 @@ int decode_scores_launch(int rows, int vocab, int dtype, const void* logits, int
                          size_t ws_bytes, cudaStream_t stream);
 size_t decode_scores_ws_bytes(int rows, int vocab);
 
+int decoder_update_launch(int B, int G, float tau_accept, float tau_remask, int32_t mask_token,
+                          const float* max_prob, const int32_t* top1, const float* cur_prob, int32_t* g,
+                          uint8_t* changed, cudaStream_t stream);
+
 int should_refresh_launch(int B, int G, const int32_t* g_cur, int32_t* g_anchor, int32_t* age,
                           int K, int max_age, int update_anchor, int32_t* dist, uint8_t* flag,
                           cudaStream_t stream);

@@ -385,3 +385,47 @@ def traj_logits(wl: Workload, seed: int, step: int):
     """Logits scored after the forward of step t: [B*G, V] bf16 bits or fp32."""
     return logits(wl.shape.batch * wl.shape.resp_len, wl.vocab, seed=seed, std=wl.logits_std,
                   boost_max=wl.logits_boost, dtype=wl.logits_dtype, step=step)
+
+
+# ----------------------------------------------------------------------------
+# closed-loop decoding: the rollback decoder D is a confidence rule on the
+# scores of the previous step's logits (oracle.decoder_update and
+# archer_decoder_update); the logits plant a per-position target token whose
+# boost grows with the step, so positions become confident at different steps
+# and early guesses that are not the target get rolled back.
+# ----------------------------------------------------------------------------
+
+# decoder thresholds and the logits' boost growth used by closed-loop runs
+CLOSED_LOOP = {"tau_accept": 0.9, "tau_remask": 0.05, "boost_per_step": 1.75}
+
+
+def closed_loop_targets(wl: Workload, seed: int = 0):
+    """Per-position target token [B, G] and boost rate [B, G] (U(0.5, 1.5))."""
+    B, G = wl.shape.batch, wl.shape.resp_len
+    u = uniform(stream_key("cl-target", seed, B, G), B * G)
+    tgt = np.minimum((u * wl.vocab).astype(np.int64), wl.vocab - 1).astype(np.int32).reshape(B, G)
+    rate = 0.5 + uniform(stream_key("cl-rate", seed, B, G), B * G).reshape(B, G)
+    return tgt, rate
+
+
+def closed_loop_logits(wl: Workload, seed: int, step: int, boost_per_step: float):
+    """Logits scored after the forward of step t: N(0, std^2) plus
+    boost_per_step * t * rate on each position's target token; bf16 bits or fp32."""
+    B, G, V = wl.shape.batch, wl.shape.resp_len, wl.vocab
+    z = normal(stream_key("cl-logits", seed, step, B, G, V), B * G * V).reshape(B * G, V) * wl.logits_std
+    tgt, rate = closed_loop_targets(wl, seed)
+    z[np.arange(B * G), tgt.reshape(-1)] += boost_per_step * step * rate.reshape(-1)
+    if wl.logits_dtype == "bf16":
+        return to_bf16_bits(z)
+    return z.astype(np.float32)
+
+
+def closed_loop_rows(wl: Workload, seed: int, step: int, layer: int) -> dict:
+    """Candidate rows for every response position at step t (a changed position
+    takes its own): q [B,G,Hq,D], k/v [B,G,Hkv,D] bf16 bits."""
+    sh = wl.shape
+    std = 1.0 / math.sqrt(sh.head_dim)
+    B, G = sh.batch, sh.resp_len
+    return {"q": bf16_normal(("cl-rows", seed, step, layer, "q"), (B, G, sh.n_heads, sh.head_dim), std),
+            "k": bf16_normal(("cl-rows", seed, step, layer, "k"), (B, G, sh.n_kv_heads, sh.head_dim), std),
+            "v": bf16_normal(("cl-rows", seed, step, layer, "v"), (B, G, sh.n_kv_heads, sh.head_dim), std)}

@@ -42,7 +42,8 @@ def _dev_bits(bits, device):
 class DeviceTrajectory:
     def __init__(self, wl: synth.Workload, seed: int = 0, mode: str = "archer", source: str = "host",
                  device="cuda", layers: int | None = None, score: bool = True, pool_steps: int = 8,
-                 max_steps: int | None = None, record: bool = False):
+                 max_steps: int | None = None, record: bool = False, decoder: str = "redraw",
+                 closed_loop: dict | None = None):
         self.wl, self.seed, self.mode, self.source = wl, seed, mode, source
         self.device = torch.device(device)
         sh = wl.shape
@@ -53,6 +54,10 @@ class DeviceTrajectory:
         if mode not in ("archer", "eager", "graph", "eager-graph"):
             raise ValueError(f"unknown mode {mode}")
         self.graph_mode = mode in ("graph", "eager-graph")
+        if decoder not in ("redraw", "closed") or (decoder == "closed" and source != "host"):
+            raise ValueError("decoder is 'redraw' or 'closed' (closed: host source only)")
+        self.closed = decoder == "closed"
+        self.cl = dict(synth.CLOSED_LOOP, **(closed_loop or {}))
         eager = mode in ("eager", "eager-graph")
         self.K = 0 if eager else wl.radius_k
         self.max_age = 0 if eager else wl.max_age
@@ -76,6 +81,8 @@ class DeviceTrajectory:
         std = 1.0 / math.sqrt(D)
         if self.source == "host":
             g0 = synth.traj_initial_tokens(self.wl, self.seed)
+            if self.closed:
+                g0 = np.full((B, G), synth.MASK_TOKEN, dtype=np.int32)
             init = [synth.traj_layer_initial(self.wl, self.seed, layer) for layer in range(L)]
             self.q_all = torch.stack([_dev_bits(x["q_all"], dev) for x in init])
             self.k_resp = torch.stack([_dev_bits(x["k_resp"], dev) for x in init])
@@ -130,6 +137,10 @@ class DeviceTrajectory:
             self.max_prob = torch.empty(rows, dtype=torch.float32, device=dev)
             self.top1 = torch.empty(rows, dtype=torch.int32, device=dev)
             self.margin = torch.empty(rows, dtype=torch.float32, device=dev)
+            if self.closed:
+                self.cur_prob = torch.empty(rows, dtype=torch.float32, device=dev)
+                self.mask_state = (self.g == synth.MASK_TOKEN).to(torch.uint8)
+                self.changed = torch.zeros(B, G, dtype=torch.uint8, device=dev)
             self.ws = A.scores_workspace(rows, V, dev)
 
     # ------------------------------------------------------------------ pieces
@@ -167,23 +178,52 @@ class DeviceTrajectory:
         if not self.score:
             return None
         self._upload_logits(t)
-        self._timed("score", lambda: A.archer_decode_scores(self.logits, self.max_prob, self.top1, self.margin,
-                                                            workspace=self.ws))
+        if self.closed:
+            self._timed("score", lambda: A.archer_decode_scores(
+                self.logits, self.max_prob, self.top1, self.margin, mask_state=self.mask_state, cur_tokens=self.g,
+                cur_prob=self.cur_prob, workspace=self.ws))
+        else:
+            self._timed("score", lambda: A.archer_decode_scores(self.logits, self.max_prob, self.top1, self.margin,
+                                                                workspace=self.ws))
         if self.record:
-            return {"max_prob": self.max_prob.clone(), "top1": self.top1.clone(), "margin": self.margin.clone()}
+            sc = {"max_prob": self.max_prob.clone(), "top1": self.top1.clone(), "margin": self.margin.clone()}
+            if self.closed:
+                sc["cur_prob"] = self.cur_prob.clone()
+            return sc
         return None
 
     def _upload_logits(self, t):
         if self.source != "host":
             return
-        z = synth.traj_logits(self.wl, self.seed, t)
+        if self.closed:
+            z = synth.closed_loop_logits(self.wl, self.seed, t, self.cl["boost_per_step"])
+        else:
+            z = synth.traj_logits(self.wl, self.seed, t)
         z = _dev_bits(z, self.device) if self.wl.logits_dtype == "bf16" else torch.from_numpy(z).to(self.device)
         if self.graph_mode:
             self.logits.copy_(z)
         else:
             self.logits = z
 
+    def _closed_loop_decode(self, t):
+        # D: the confidence rule on the previous step's scores, on the device;
+        # every position's candidate rows are uploaded, the changed ones kept
+        A.archer_decoder_update(self.g, self.max_prob, self.top1, self.cur_prob, self.changed,
+                                self.cl["tau_accept"], self.cl["tau_remask"], synth.MASK_TOKEN)
+        self.mask_state.copy_((self.g == synth.MASK_TOKEN).to(torch.uint8))
+        ch = self.changed.bool()[:, :, None, None]
+        P = self.P
+        for layer in range(self.L):
+            rows = synth.closed_loop_rows(self.wl, self.seed, t, layer)
+            q, k, v = (_dev_bits(rows[c], self.device) for c in ("q", "k", "v"))
+            self.q_resp[layer].copy_(torch.where(ch, q, self.q_resp[layer]))
+            self.q_all[layer][:, P:] = torch.where(ch, q, self.q_all[layer][:, P:])
+            self.k_resp[layer].copy_(torch.where(ch, k, self.k_resp[layer]))
+            self.v_resp[layer].copy_(torch.where(ch, v, self.v_resp[layer]))
+
     def _stage_redraw(self, t):
+        if self.closed:
+            return self._closed_loop_decode(t)
         B, P = self.B, self.P
         if self.wl.redraws_per_step == 0:
             return
@@ -249,6 +289,8 @@ class DeviceTrajectory:
         if self.score:
             sc = dict(logits=self.logits, max_prob=self.max_prob, top1=self.top1, margin=self.margin,
                       workspace=self.ws)
+            if self.closed:
+                sc.update(mask_state=self.mask_state, cur_tokens=self.g, cur_prob=self.cur_prob)
         self.refresh_count.zero_()
         self.graph = A.StepGraph(self.shape, layers, self.g, self.g_anchor, self.age, self.K, self.max_age,
                                  self.flag, dist_out=self.dist, refresh_count=self.refresh_count, **sc)
@@ -268,9 +310,11 @@ class DeviceTrajectory:
             refreshed = bool(flags.any())
             # the layers share one output buffer: only the last layer's survives the replay
             outs = [None] * (self.L - 1) + [(self.out_full if refreshed else self.out_step).clone()]
-            rec.update({"flag": flags, "out": outs, "dist": self.dist.cpu().numpy(),
-                        "scores": {"max_prob": self.max_prob.clone(), "top1": self.top1.clone(),
-                                   "margin": self.margin.clone()} if self.score else None})
+            rec.update({"flag": flags, "out": outs, "dist": self.dist.cpu().numpy(), "g": self.g.cpu().numpy(),
+                        "scores": ({"max_prob": self.max_prob.clone(), "top1": self.top1.clone(),
+                                    "margin": self.margin.clone(),
+                                    **({"cur_prob": self.cur_prob.clone()} if self.closed else {})}
+                                   if self.score else None)})
         return rec
 
     def step(self):
@@ -291,6 +335,7 @@ class DeviceTrajectory:
         rec = {"t": t, "flag": flags.copy(), "out": outs, "scores": sc}
         if self.record:
             rec["dist"] = self.dist.cpu().numpy()
+            rec["g"] = self.g.cpu().numpy()
         return rec
 
     def attention_flops(self, refresh: bool) -> float:

@@ -94,3 +94,13 @@ def test_step_graph_arguments_rejected_before_any_cuda_call(lib):
     assert lib.archer_step_graph_launch(None, None) == -1
     lib.archer_step_graph_destroy.argtypes = [ctypes.c_void_p]
     assert lib.archer_step_graph_destroy(None) == 0
+
+
+def test_decoder_update_arguments_rejected(lib):
+    f = lib.archer_decoder_update
+    f.argtypes = [ctypes.c_int, ctypes.c_int, ctypes.c_float, ctypes.c_float, ctypes.c_int32] + [ctypes.c_void_p] * 6
+    p = ctypes.c_void_p(0x10000)
+    assert f(-1, 4, 0.9, 0.05, -1, p, p, p, p, p, None) == -1
+    assert f(2, 4, 0.9, 0.05, -1, None, p, p, p, p, None) == -1
+    assert f(2, 4, float("nan"), 0.05, -1, p, p, p, p, p, None) == -1
+    assert f(0, 4, 0.9, 0.05, -1, None, None, None, None, None, None) == 0

@@ -95,3 +95,60 @@ def test_step_graph_equals_host_driven_steps_bit_for_bit():
         for k in ("max_prob", "top1", "margin"):
             assert torch.equal(ra["scores"][k], rg["scores"][k])
     assert a.n_refresh_steps == g.n_refresh_steps
+
+
+def _closed_workload():
+    import dataclasses
+    return dataclasses.replace(synth.WORKLOADS["tiny"], radius_k=8, max_age=0, steps=10)
+
+
+def _decision_gap(recs, cl):
+    """Smallest distance of an oracle decision quantity to its threshold (and,
+    on steps where the progress rule decides, of the best masked probability
+    to the runner-up)."""
+    gap = np.inf
+    for r in recs[:-1]:
+        g, sc = r["g"].reshape(-1), r["scores"]
+        masked = g == synth.MASK_TOKEN
+        if masked.any():
+            mpm = sc["max_prob"][masked]
+            gap = min(gap, np.abs(mpm - cl["tau_accept"]).min())
+            if (mpm < cl["tau_accept"]).all() and len(mpm) > 1:
+                top = np.sort(mpm)[::-1]
+                if top[0] > top[1]:
+                    gap = min(gap, top[0] - top[1])
+        if (~masked).any():
+            gap = min(gap, np.abs(sc["cur_prob"][~masked] - cl["tau_remask"]).min())
+    return gap
+
+
+@pytest.mark.parametrize("dev_mode", ["archer", "graph"])
+def test_closed_loop_decoder_trajectory_matches_oracle(dev_mode):
+    # The decoder's choices read the scoring kernel's outputs, so the refresh
+    # flags now depend on them: tokens, flags, outputs and scores must match the
+    # oracle's closed loop step by step.
+    from paper_2608_08086_gb300.trajectory import DeviceTrajectory
+    wl = _closed_workload()
+    cl = synth.CLOSED_LOOP
+    seed = 24         # refreshes at t = 6, 8, 10 between cached steps; no decision near a threshold
+    ref = OT.run(wl, seed=seed, decoder="closed")
+    assert _decision_gap(ref, cl) > 2e-4, "seed chosen so that no decision sits within tolerance of a threshold"
+    tr = DeviceTrajectory(wl, seed=seed, mode=dev_mode, source="host", record=True, decoder="closed")
+    got = [tr.build()] + [tr.step() for _ in range(wl.steps)]
+    torch.cuda.synchronize()
+    assert any(r["flag"].any() for r in ref[1:]), "the distance rule should fire"
+    for r, g in zip(ref, got):
+        t = r["t"]
+        if t > 0:
+            np.testing.assert_array_equal(g["g"], r["g"], err_msg=f"tokens at step {t}")
+            np.testing.assert_array_equal(g["flag"], r["flag"], err_msg=f"flags at step {t}")
+        o_ref, o_got = r["out"][-1], g["out"][-1]
+        o_got = _host(o_got)
+        err = np.abs(o_got - o_ref) - (2e-2 + 2e-2 * np.abs(o_ref))
+        assert (err <= 0).all(), f"attention at step {t}"
+        s_ref, s_got = r["scores"], {k: v.cpu().numpy() for k, v in g["scores"].items()}
+        keep = s_ref["margin"] >= 1e-4
+        assert (s_got["top1"][keep] == s_ref["top1"][keep]).all(), f"top-1 at step {t}"
+        for k in ("max_prob", "margin", "cur_prob"):
+            err = np.abs(s_got[k] - s_ref[k]) - (1e-5 + 1e-4 * np.abs(s_ref[k]))
+            assert (err <= 0).all(), f"{k} at step {t}"
