@@ -317,6 +317,52 @@ def sweep(args):
     return 0
 
 
+def staleness(args):
+    """The staleness curve of a cached step (Eq. theory-radius-bound) on a
+    LLaDA-shaped layer (B1, 32 heads, D128, P512, G256) whose prompt cache is
+    the linear synthetic map of synth.staleness_model: the CUDA cached step
+    against K_p(g_r) and against K_p(g_t) at Hamming distance D (caches in
+    bf16), err = max |O_cached - O_fresh|, and the bound Gamma sqrt(D) of that
+    map (one JSON line per D)."""
+    from paper_2608_08086_gb300 import archer as A
+    shape = synth.AttnShape(1, 512, 256, 32, 32, 128)
+    B, P, G, Hq, Hkv, D = 1, 512, 256, 32, 32, 128
+    m = synth.staleness_model(shape, seed=0)
+    scale = 1.0 / math.sqrt(D)
+    dev = torch.device("cuda")
+
+    def dev_bits(bits):
+        return torch.from_numpy(np.ascontiguousarray(bits).view(np.int16)).view(torch.bfloat16).to(dev)
+
+    g_r = synth.staleness_tokens(0, B, G)
+    kc, vc = synth.staleness_prompt_cache(m, g_r, Hkv, D)
+    kc_b, vc_b = synth.to_bf16_bits(kc), synth.to_bf16_bits(vc)
+    q, kg, vg = dev_bits(m["q_resp"]), dev_bits(m["k_resp"]), dev_bits(m["v_resp"])
+    sh = A.make_shape(B, P, G, Hq, Hkv, D)
+    # Gamma = B_e max_j ||alpha_j|| (||A_V|| + s max ||q|| ||A_K|| max |v|)  (L_Phi L_C B)
+    emb = m["emb"]
+    b_e = float(np.sqrt(((emb[:, None] - emb[None]) ** 2).sum(-1)).max())
+    f64 = synth.bf16_bits_to_f64
+    qn = float(np.linalg.norm(f64(m["q_resp"]), axis=-1).max())
+    vmax = max(float(np.abs(f64(vc_b)).max()), float(np.abs(f64(m["v_resp"])).max()))
+    gam = b_e * float(np.linalg.norm(m["alpha"], axis=1).max()) * (
+        float(np.linalg.norm(m["a_v"], 2)) + scale * qn * float(np.linalg.norm(m["a_k"], 2)) * vmax)
+
+    def run(kb, vb):
+        out = torch.empty(B, G, Hq, D, dtype=torch.bfloat16, device=dev)
+        A.archer_attn_step(sh, q, dev_bits(kb), dev_bits(vb), kg, vg, out)
+        return out.float()
+
+    o_cached = run(kc_b, vc_b)
+    for d in (0, 1, 2, 4, 8, 16, 32, 64, 128, 256):
+        kf, vf = synth.staleness_prompt_cache(m, synth.staleness_drift(g_r, d, 0), Hkv, D)
+        err = float((run(synth.to_bf16_bits(kf), synth.to_bf16_bits(vf)) - o_cached).abs().max())
+        print(json.dumps({"staleness": "llada_layer", "D_t": d, "err_inf": err, "gamma_sqrt_d": gam * math.sqrt(d),
+                          "err_over_sqrt_d": err / math.sqrt(d) if d else 0.0, "gamma": gam}), flush=True)
+    A.archer_check_device()
+    return 0
+
+
 def kernel_stats(tr):
     """Mean durations (ms) and counts of the attention / scoring launches."""
     by = {}
@@ -520,6 +566,8 @@ def main():
     ap.add_argument("--kernel-only", choices=["attn_step", "attn_refresh", "scores"], default=None,
                     help="run only a few launches of one kernel (for profiler captures)")
     ap.add_argument("--launches", type=int, default=3)
+    ap.add_argument("--staleness", action="store_true",
+                    help="staleness curve of a cached step against the Hamming distance (Eq. theory-radius-bound)")
     ap.add_argument("--sweep", action="store_true",
                     help="per-configuration measurements (LLaDA layer, scoring, prompt-length sweep)")
     args = ap.parse_args()
@@ -528,10 +576,12 @@ def main():
 
     if args.impl == "reference":
         return reference_arm(args, wl)
-    if args.kernel_only or args.sweep:
+    if args.kernel_only or args.sweep or args.staleness:
         torch.cuda.set_device(int(os.environ.get("LOCAL_RANK", "0")))
         from paper_2608_08086_gb300 import build as Bld
         Bld.build()
+        if args.staleness:
+            return staleness(args)
         return sweep(args) if args.sweep else kernel_only(args, wl)
 
     world = int(os.environ.get("WORLD_SIZE", "1"))

@@ -429,3 +429,63 @@ def closed_loop_rows(wl: Workload, seed: int, step: int, layer: int) -> dict:
     return {"q": bf16_normal(("cl-rows", seed, step, layer, "q"), (B, G, sh.n_heads, sh.head_dim), std),
             "k": bf16_normal(("cl-rows", seed, step, layer, "k"), (B, G, sh.n_kv_heads, sh.head_dim), std),
             "v": bf16_normal(("cl-rows", seed, step, layer, "v"), (B, G, sh.n_kv_heads, sh.head_dim), std)}
+
+
+# ----------------------------------------------------------------------------
+# staleness experiment: a synthetic prompt-cache map C_p(g) that is linear in
+# the response embeddings E(g), so that Eq. theory-smoothness holds with a
+# known constant:  K_p(g) = K_0 + alpha E(g) A_K^T,  V_p(g) = V_0 + alpha E(g) A_V^T
+# (alpha [P, G], E(g) [G, d_e] one unit-norm embedding per token id, A [Hkv D, d_e]).
+# ----------------------------------------------------------------------------
+
+def staleness_model(shape: AttnShape, seed: int = 0, n_tokens: int = 64, d_e: int = 16,
+                    drift: float = 0.6) -> dict:
+    """Random pieces of the linear prompt-cache map (fp64) plus the layer's
+    response queries and K/V (bf16 bits).  n_tokens embeddings (the last one is
+    MASK_TOKEN's), rows normalised to 1; alpha ~ N(0, 1/G), A ~ N(0, 1/d_e),
+    scaled by drift / sqrt(D) so that changing every position moves K_p by
+    about drift times the spread of K_0."""
+    B, P, G, Hq, Hkv, D = (shape.batch, shape.prompt_len, shape.resp_len, shape.n_heads, shape.n_kv_heads,
+                           shape.head_dim)
+    emb = normal(stream_key("st-emb", seed, n_tokens, d_e), n_tokens * d_e).reshape(n_tokens, d_e)
+    emb /= np.linalg.norm(emb, axis=1, keepdims=True)
+    alpha = normal(stream_key("st-alpha", seed, P, G), P * G).reshape(P, G) / math.sqrt(G)
+    c = drift / math.sqrt(D)
+    a_k = normal(stream_key("st-ak", seed, Hkv, D, d_e), Hkv * D * d_e).reshape(Hkv * D, d_e) * c / math.sqrt(d_e)
+    a_v = normal(stream_key("st-av", seed, Hkv, D, d_e), Hkv * D * d_e).reshape(Hkv * D, d_e) * c / math.sqrt(d_e)
+    x = attn_inputs(shape, seed=seed)
+    return {"emb": emb, "alpha": alpha, "a_k": a_k, "a_v": a_v,
+            "k0": bf16_bits_to_f64(x["k_cache"]), "v0": bf16_bits_to_f64(x["v_cache"]),
+            "q_resp": x["q_all"][:, P:], "k_resp": x["k_resp"], "v_resp": x["v_resp"]}
+
+
+def staleness_tokens(seed: int, batch: int, resp_len: int, n_tokens: int = 64) -> np.ndarray:
+    """Anchor response g_r [B, G]: ids in [0, n_tokens - 1) (the last id is MASK's)."""
+    u = uniform(stream_key("st-g", seed, batch, resp_len), batch * resp_len)
+    return np.minimum((u * (n_tokens - 1)).astype(np.int64), n_tokens - 2).reshape(batch, resp_len)
+
+
+def staleness_drift(g_r: np.ndarray, n_changed: int, seed: int, n_tokens: int = 64) -> np.ndarray:
+    """g_t at Hamming distance n_changed from g_r in every sequence.  The drift
+    is nested: a fixed seeded order of positions and a fixed new id per
+    position (another id, uniform over the remaining ones); distance D changes
+    the first D positions of that order."""
+    B, G = g_r.shape
+    g = g_r.copy()
+    for b in range(B):
+        u = raw64(stream_key("st-pos", seed, b), 0, G)
+        pos = np.argsort(u, kind="stable")[:n_changed]
+        v = uniform(stream_key("st-new", seed, b), G)[pos]
+        shift = 1 + np.minimum((v * (n_tokens - 1)).astype(np.int64), n_tokens - 2)
+        g[b, pos] = (g[b, pos] + shift) % n_tokens
+    return g
+
+
+def staleness_prompt_cache(model: dict, g: np.ndarray, Hkv: int, D: int):
+    """K_p(g), V_p(g) [B, P, Hkv, D] in fp64 (the exact map; callers round to
+    bf16 where the kernels need bf16)."""
+    ae = np.einsum("pg,bge->bpe", model["alpha"], model["emb"][g])      # [B, P, d_e]
+    dk = np.einsum("bpe,ce->bpc", ae, model["a_k"])
+    dv = np.einsum("bpe,ce->bpc", ae, model["a_v"])
+    B, P = g.shape[0], model["alpha"].shape[0]
+    return (model["k0"] + dk.reshape(B, P, Hkv, D), model["v0"] + dv.reshape(B, P, Hkv, D))
