@@ -9,7 +9,7 @@
 // formed in memory.  GQA: query head h reads KV head h / (Hq / Hkv).
 //
 // One CTA = two 128-row query tiles (A and B) of one (b, h) sharing every K/V
-// tile; 18 warps:
+// tile; 10 warps:
 //   warp 0     MMA issuer: the warp waits together, lane 0 issues.  Per K/V
 //              tile j: PV_A(j), QK_A(j+1), PV_B(j), QK_B(j+1), so the tensor
 //              pipe works on one tile while the other tile's softmax runs.  It
@@ -24,16 +24,16 @@
 //              128-key tiles (u = 0 .. T; the first pair holds K_0 only, the
 //              last V_{T-1} only) through two pair slots, one full and one
 //              empty barrier per pair.
-//   warps 2-17 softmax: four groups of four consecutive warps, (tile A, keys
-//              0-63), (A, 64-127), (B, 0-63), (B, 64-127).  Warp w reaches TMEM
-//              lanes 32 (w % 4) .. 32 (w % 4) + 31, so lane i of warp w owns
-//              query row 32 (w % 4) + i for its 64 key columns, read from TMEM
-//              once per tile.  The two groups of a tile exchange their row
-//              maxima through shared memory (a named barrier per tile);
-//              exponentials use the running max in use, raised lazily (only
-//              when the tile max exceeds it by more than 2^8, rescaling l and
-//              each group's half of O).  Each group writes its half of P (bf16
-//              pairs) over the first 32 of its own 64 S columns.
+//   warps 2-9  softmax: one warpgroup per tile.  Warp w reaches TMEM lanes
+//              32 (w % 4) .. 32 (w % 4) + 31, so lane i of warp w owns query
+//              row 32 (w % 4) + i and all 128 key columns of its tile, read
+//              from TMEM once per tile; exponentials use the running max in
+//              use, raised lazily (only when the tile max exceeds it by more
+//              than 2^8, rescaling l and O); P (bf16 pairs) is written over S
+//              columns already read.  (Two warpgroups per tile, each with half
+//              the columns and a shared-memory max exchange, measured 3 %
+//              slower: the extra warps' waiting and exchange cost the MMA warp
+//              more issue slots than the shorter rows saved.)
 // TMEM (512 columns): S_A [0,128) S_B [128,256) O_A [256,256+D) O_B [384,384+D).
 // Every hand-off is an mbarrier; every wait is bounded (archer_device.cuh).
 
@@ -53,7 +53,7 @@ namespace {
 
 constexpr int kBM = 128;          // query rows per tile (tcgen05 M)
 constexpr int kBN = 128;          // keys per KV tile (N of Q K^T, K of P V)
-constexpr int kThreads = 576;     // 4 softmax warpgroups + producer warp + MMA warp
+constexpr int kThreads = 320;     // MMA warp + producer warp + 2 softmax warpgroups
 constexpr int kWarpMma = 0, kWarpProducer = 1, kWarpSoftmax0 = 2;
 constexpr uint32_t kTmemCols = 512;
 // TMEM columns of tile t's S (P is written over its first 64 columns) and O.
@@ -91,8 +91,7 @@ struct Layout {
   static constexpr uint32_t kOffBar = kOffKV + kSlots * 2 * kTile;
   // q_full, full[slots], empty[slots], s_full[2], p_full[2]
   static constexpr int kBars = 1 + 2 * kSlots + 4;
-  static constexpr uint32_t kOffXch = kOffBar + 8 * kBars;  // [tile parity][tile][half][row] floats
-  static constexpr uint32_t kOffHolder = kOffXch + 2 * 2 * 2 * 128 * 4;
+  static constexpr uint32_t kOffHolder = kOffBar + 8 * kBars;
   static constexpr uint32_t kOffAbort = kOffHolder + 4;
   static constexpr uint32_t kUsed = kOffAbort + 4;
   // + 1 KB to align the base to 1024 B; at least 120 KB so that one CTA
@@ -118,11 +117,6 @@ __device__ __forceinline__ bool warp_wait(uint32_t bar, uint32_t parity, volatil
       return false;
     }
   }
-}
-
-// Named barrier for the 256 softmax threads of tile t (ids 1 and 2; 0 is __syncthreads).
-__device__ __forceinline__ void tile_bar(int t) {
-  asm volatile("bar.sync %0, 256;" ::"r"(1 + t) : "memory");
 }
 
 __device__ __forceinline__ float max3f(float a, float b, float c) {
@@ -151,23 +145,23 @@ __device__ __forceinline__ float2 fadd2(float2 a, float2 b) {
   return d;
 }
 
-__device__ __forceinline__ float max64(const float (&x)[64]) {
+__device__ __forceinline__ float max128(const float (&x)[128]) {
   float m[4] = {x[0], x[1], x[2], x[3]};
 #pragma unroll
-  for (int c = 4; c < 64; c += 2) m[(c >> 1) & 3] = max3f(m[(c >> 1) & 3], x[c], x[c + 1]);
+  for (int c = 4; c < 128; c += 2) m[(c >> 1) & 3] = max3f(m[(c >> 1) & 3], x[c], x[c + 1]);
   return max3f(m[0], m[1], fmaxf(m[2], m[3]));
 }
 
-// Loads 64 score columns [c0, c0 + 64) of this lane and masks keys >= valid.
-__device__ __forceinline__ void load_scores64(uint32_t taddr, int c0, int valid, float (&x)[64]) {
-  uint32_t r[64];
-  tmem_ld_64(taddr, r);
+// Loads this lane's 128 score columns and masks keys >= valid.
+__device__ __forceinline__ void load_scores128(uint32_t taddr, int valid, float (&x)[128]) {
+  uint32_t r[128];
+  tmem_ld_128(taddr, r);
 #pragma unroll
-  for (int c = 0; c < 64; ++c) x[c] = __uint_as_float(r[c]);
-  if (valid < c0 + 64) {            // only the last tile of a segment is ragged
+  for (int c = 0; c < 128; ++c) x[c] = __uint_as_float(r[c]);
+  if (valid < 128) {                // only the last tile of a segment is ragged
 #pragma unroll
-    for (int c = 0; c < 64; ++c)
-      if (c0 + c >= valid) x[c] = -INFINITY;
+    for (int c = 0; c < 128; ++c)
+      if (c >= valid) x[c] = -INFINITY;
   }
 }
 
@@ -209,7 +203,6 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
   const uint32_t bar_empty = bar_full + 8 * L::kSlots;          // + 8 * slot
   const uint32_t bar_s_full = bar_empty + 8 * L::kSlots;        // + 8 * tile (A = 0, B = 1)
   const uint32_t bar_p_full = bar_s_full + 16;                  // + 8 * tile: both halves of P written
-  float* xch = reinterpret_cast<float*>(gbase + L::kOffXch);
   uint32_t* holder = reinterpret_cast<uint32_t*>(gbase + L::kOffHolder);
   volatile int* abort = reinterpret_cast<volatile int*>(gbase + L::kOffAbort);
 
@@ -222,7 +215,7 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
     }
     for (int i = 0; i < 2; ++i) {
       mbar_init(bar_s_full + 8 * i, 1);
-      mbar_init(bar_p_full + 8 * i, 2 * kBM);
+      mbar_init(bar_p_full + 8 * i, kBM);
     }
     *abort = 0;
     mbar_fence_init();
@@ -330,53 +323,42 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
     }
   } else {
     // ------------------------------------------------------------ softmax
-    const int sw = warp - kWarpSoftmax0;
-    const int t = sw >> 3;                                        // 0 = tile A, 1 = tile B
-    const int c = (sw >> 2) & 1;                                  // key half: columns [64c, 64c + 64)
+    const int t = (warp - kWarpSoftmax0) >> 2;                    // 0 = tile A, 1 = tile B
     if (t == 0 || has_b) {
-      const int r = (warp & 3) * 32 + (threadIdx.x & 31);         // query row in the tile = TMEM lane
+      const int r = (warp & 3) * 32 + (threadIdx.x & 31);
       const uint32_t t_lane = tmem + (static_cast<uint32_t>((warp & 3) * 32) << 16);
       const uint32_t colS = col_s(t), colO = col_o(t);
       const uint32_t bar_s = bar_s_full + 8 * t;
       const uint32_t bar_ph = bar_p_full + 8 * t;
-      // exchange slots, double-buffered by tile parity: slot(par, group)
-      auto slot = [&](int par, int grp) { return xch + ((par * 2 + t) * 2 + grp) * 128; };
       const float sl2 = p.scale_log2;
-      float m_used = -INFINITY;                                  // running max in use (log2 units)
-      float2 l2 = make_float2(0.f, 0.f);                         // this half's row sum, two lanes
-      // O *= a over this group's half of the O columns (16 at a time: the
-      // tile's 64 scores stay in registers meanwhile)
+      float m_used = -INFINITY;
+      float2 l2 = make_float2(0.f, 0.f);
+      // O *= a, 16 columns at a time (the row's scores stay in registers)
       auto rescale_o = [&](float a) {
 #pragma unroll 1
-        for (int c0 = 0; c0 < D / 2; c0 += 16) {
+        for (int c0 = 0; c0 < D; c0 += 16) {
           uint32_t o[16];
-          tmem_ld_16(t_lane + colO + c * (D / 2) + c0, o);
+          tmem_ld_16(t_lane + colO + c0, o);
 #pragma unroll
           for (int k = 0; k < 16; ++k) o[k] = __float_as_uint(__uint_as_float(o[k]) * a);
-          tmem_st_16(t_lane + colO + c * (D / 2) + c0, o);
+          tmem_st_16(t_lane + colO + c0, o);
         }
       };
-      // An expired wait sets the abort flag; the groups then run on over stale
-      // TMEM (in bounds) so that both groups of a tile meet every named barrier.
+      // An expired wait sets the abort flag; the warps then run on over stale
+      // TMEM (in bounds) to the epilogue.
       for (int j = 0; j < T; ++j) {
         warp_wait(bar_s, j & 1, abort, p.err, p.wait_limit);
         tc_fence_after();
-        const int jg = j0 + j;                                    // global key tile
+        const int jg = j0 + j;
         const int valid = jg < n_p ? min(kBN, p.P - jg * kBN) : min(kBN, p.G - (jg - n_p) * kBN);
-        // The group's 64 scores are read from TMEM once and kept in registers.
-        float x[64];
-        load_scores64(t_lane + colS + 64 * c, 64 * c, valid, x);
-        const float hm = max64(x);
-        // A slot of parity j & 1 is rewritten at tile j + 2 only after both
-        // groups passed tile j + 1's barrier, i.e. after it was read.
-        slot(j & 1, c)[r] = hm * sl2;
-        tile_bar(t);                       // both halves' maxima published
-        const float tm = fmaxf(slot(j & 1, c)[r], slot(j & 1, c ^ 1)[r]);
+        // The row's 128 scores are read from TMEM once and kept in registers.
+        float x[128];
+        load_scores128(t_lane + colS, valid, x);
+        const float tm = max128(x) * sl2;
         if (j == 0) {
           m_used = tm;
         } else if (__any_sync(0xffffffffu, tm > m_used + 8.0f)) {
-          // Same rows, same maxima in both groups: the same decision.  O holds
-          // P V up to tile j-1, complete (S(j) was announced after it).
+          // O holds P V up to tile j-1, complete (S(j) was announced after it).
           const float m_new = fmaxf(m_used, tm);
           const float a = ex2_approx(m_used - m_new);
           m_used = m_new;
@@ -387,42 +369,39 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
         const float2 neg_m = make_float2(-m_used, -m_used);
         const float2 slv = make_float2(sl2, sl2);
         float2 acc[2] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
-        uint32_t pk[2][16];
 #pragma unroll
-        for (int q32 = 0; q32 < 2; ++q32) {
+        for (int q = 0; q < 4; ++q) {
+          // P of keys [32q, 32q + 32) as bf16 pairs over S columns that were
+          // already read: keys [64h, 64h + 64) go to columns [64h, 64h + 32),
+          // the layout the MMA warp's P V reads; each store stays in flight
+          // while the next chunk is computed.
+          uint32_t pk[16];
 #pragma unroll
           for (int k = 0; k < 16; ++k) {
-            const float2 y = ffma2(make_float2(x[32 * q32 + 2 * k], x[32 * q32 + 2 * k + 1]), slv, neg_m);
+            const float2 y = ffma2(make_float2(x[32 * q + 2 * k], x[32 * q + 2 * k + 1]), slv, neg_m);
             const float2 pr = make_float2(ex2_approx(y.x), ex2_approx(y.y));
             acc[k & 1] = fadd2(acc[k & 1], pr);
-            pk[q32][k] = pack_bf16x2(pr.x, pr.y);
+            pk[k] = pack_bf16x2(pr.x, pr.y);
           }
-          // P over the first 32 of this group's own S columns (all 64 already
-          // read); the store stays in flight while the next chunk is computed.
-          tmem_st_16_async(t_lane + colS + 64 * c + 16 * q32, pk[q32]);
+          tmem_st_16_async(t_lane + colS + 64 * (q >> 1) + 16 * (q & 1), pk);
         }
         tmem_wait_st();
         l2 = fadd2(l2, fadd2(acc[0], acc[1]));
         tc_fence_before();
         mbar_arrive(bar_ph);
       }
-      // epilogue: combine the two halves' row sums, normalise this half of O
       const bool ok = warp_wait(bar_s, T & 1, abort, p.err, p.wait_limit);
       tc_fence_after();
-      tile_bar(t);                         // every exchange slot has been read
-      slot(0, c)[r] = l2.x + l2.y;
-      tile_bar(t);
-      const float l_sum = slot(0, c)[r] + slot(0, c ^ 1)[r];
+      const float l_sum = l2.x + l2.y;
       const int q = q0 + t * kBM + r;
       const bool live = ok && q < p.M;
       if (partial) {
-        // unnormalised O, max and sum of this key range, merged by the combine kernel
         const size_t row = ((static_cast<size_t>(split) * gridDim.z + b) * p.Hq + h) * p.M + q;
-        float* orow_ws = p.ws_o + row * D + c * (D / 2);
+        float* orow_ws = p.ws_o + row * D;
 #pragma unroll
-        for (int c0 = 0; c0 < D / 2; c0 += 32) {
+        for (int c0 = 0; c0 < D; c0 += 32) {
           uint32_t o[32];
-          tmem_ld_32(t_lane + colO + c * (D / 2) + c0, o);
+          tmem_ld_32(t_lane + colO + c0, o);
           if (live) {
             float4* dst = reinterpret_cast<float4*>(orow_ws + c0);
 #pragma unroll
@@ -431,14 +410,14 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
                                    __uint_as_float(o[4 * v + 2]), __uint_as_float(o[4 * v + 3]));
           }
         }
-        if (live && c == 0) p.ws_ml[row] = make_float2(m_used, l_sum);
+        if (live) p.ws_ml[row] = make_float2(m_used, l_sum);
       } else {
         const float inv_l = 1.0f / l_sum;
-        __nv_bfloat16* orow = p.out + ((static_cast<size_t>(b) * p.M + q) * p.Hq + h) * D + c * (D / 2);
+        __nv_bfloat16* orow = p.out + ((static_cast<size_t>(b) * p.M + q) * p.Hq + h) * D;
 #pragma unroll
-        for (int c0 = 0; c0 < D / 2; c0 += 32) {
+        for (int c0 = 0; c0 < D; c0 += 32) {
           uint32_t o[32];
-          tmem_ld_32(t_lane + colO + c * (D / 2) + c0, o);
+          tmem_ld_32(t_lane + colO + c0, o);
           uint32_t w[16];
 #pragma unroll
           for (int k = 0; k < 16; ++k)
@@ -449,7 +428,7 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
             for (int v = 0; v < 4; ++v) dst[v] = make_uint4(w[4 * v], w[4 * v + 1], w[4 * v + 2], w[4 * v + 3]);
           }
         }
-        if (live && c == 0 && p.lse)
+        if (live && p.lse)
           p.lse[(static_cast<size_t>(b) * p.Hq + h) * p.M + q] = (m_used + log2f(l_sum)) * 0.69314718055994531f;
       }
     }
