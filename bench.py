@@ -424,10 +424,7 @@ def run_e2e(wl, steps, warmup, dist_on, seed=0):
         pos, new = d_plan[slot]
         bidx = torch.arange(B, device=tr.device)[:, None]
         tr.g[bidx, pos] = new
-        tr.q_resp[:, bidx, pos] = d_rows[slot]["q"]
-        tr.q_all[:, bidx, P + pos] = d_rows[slot]["q"]
-        tr.k_resp[:, bidx, pos] = d_rows[slot]["k"]
-        tr.v_resp[:, bidx, pos] = d_rows[slot]["v"]
+        tr._scatter(d_rows[slot]["q"], d_rows[slot]["k"], d_rows[slot]["v"], pos)
         tr.logits = d_logits[slot]
 
     fresh_stream = torch.cuda.Stream()
@@ -622,8 +619,9 @@ def main():
     host_value = world * args.steps / (max_over_ranks(arm["ms"], dist_on) / 1e3)
     ks = kernel_stats(tr)
     L = tr.L
-    # per step: rule + refresh condition + L attention + scoring (2) [+ L cache rewrites on refresh steps]
-    launches = args.steps * (2 + L + (2 if tr.score else 0)) + n_ref * L
+    # per step: 3 row scatters + rule + refresh condition + L attention + scoring (2)
+    # [+ L cache rewrites on refresh steps]
+    launches = args.steps * (3 + 2 + L + (2 if tr.score else 0)) + n_ref * L
     flops_step_launch = 4.0 * tr.B * tr.Hq * tr.G * tr.N * tr.D
     flops_refresh_launch = 4.0 * tr.B * tr.Hq * tr.N * tr.N * tr.D
     att = {}

@@ -197,6 +197,22 @@ int archer_decoder_update(int batch, int resp_len, float tau_accept, float tau_r
                           int32_t mask_token, const float* max_prob, const int32_t* top1,
                           const float* cur_prob, int32_t* g, uint8_t* changed, void* stream);
 
+/*
+ * Row scatter (staging, no counterpart in the paper's method): puts a step's
+ * new response rows -- the Q, K or V rows of the positions the decoder
+ * changed, for every layer -- into the layer tensors.  For o < n_outer,
+ * b < batch, r < n, the row_bytes bytes at
+ *   src + ((o * batch + b) * n + r) * row_bytes
+ * are copied to
+ *   dst0 + ((o * batch + b) * dst0_rows + dst0_row0 + pos[b * n + r]) * row_bytes
+ * and, when dst1 is not NULL, likewise to dst1 (dst1_rows, dst1_row0).
+ * pos [batch, n] int64; a position outside [0, dst_rows - dst_row0) is
+ * skipped.  row_bytes a multiple of 16; pointers 16-byte aligned.
+ */
+int archer_scatter_rows(int n_outer, int batch, int n, size_t row_bytes, const void* src,
+                        const int64_t* pos, void* dst0, int dst0_rows, int dst0_row0, void* dst1,
+                        int dst1_rows, int dst1_row0, void* stream);
+
 /* Bit-exact copy of a refreshed sequence's prompt K/V into the cache
  * (the cache rewrite C_r <- C_p(g_t) of Algorithm 1) for sequences whose flag
  * is set (all when flags is NULL).  src/dst [B, P, Hkv, D] bf16. */

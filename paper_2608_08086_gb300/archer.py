@@ -74,6 +74,7 @@ def _load():
     L.archer_decode_scores_workspace_size.restype = sz
     L.archer_should_refresh.argtypes = [i, i, vp, vp, vp, i, i, i, vp, vp, vp]
     L.archer_cache_rewrite.argtypes = [sp, vp, vp, vp, vp, vp, vp]
+    L.archer_scatter_rows.argtypes = [i, i, i, sz, vp, vp, vp, i, i, vp, i, i, vp]
     L.archer_decoder_update.argtypes = [i, i, ctypes.c_float, ctypes.c_float, ctypes.c_int32, vp, vp, vp, vp, vp,
                                         vp]
     L.archer_check_device.argtypes = [vp]
@@ -87,7 +88,7 @@ def _load():
     L.archer_step_graph_destroy.argtypes = [vp]
     for name in ("archer_attn_step", "archer_prompt_refresh", "archer_decode_scores", "archer_should_refresh",
                  "archer_cache_rewrite", "archer_check_device", "archer_version", "archer_step_graph_create",
-                 "archer_decoder_update",
+                 "archer_decoder_update", "archer_scatter_rows",
                  "archer_step_graph_launch", "archer_step_graph_destroy"):
         getattr(L, name).restype = ctypes.c_int
     return L
@@ -295,6 +296,22 @@ def archer_decoder_update(g, max_prob, top1, cur_prob, changed, tau_accept, tau_
                                      _ptr(max_prob, None, "max_prob"), _ptr(top1, None, "top1"),
                                      _ptr(cur_prob, None, "cur_prob"), _ptr(g, torch.int32, "g"),
                                      _ptr(changed, torch.uint8, "changed"), _stream(stream)))
+
+
+def archer_scatter_rows(src, pos, dst0, dst0_row0=0, dst1=None, dst1_row0=0, stream=None):
+    """Row scatter (see include/archer.h): src [O, B, n, *row], pos [B, n] int64,
+    dst [O, B, rows, *row] (same row shape); rows of dst0 / dst1 start at
+    dst*_row0."""
+    O, B, n = src.shape[:3]
+    row = src[0, 0, 0].numel() * src.element_size() if src.numel() else 0
+    for d, name in ((dst0, "dst0"), (dst1, "dst1")):
+        if d is not None and (tuple(d.shape[:2]) != (O, B) or d[0, 0, 0].numel() * d.element_size() != row):
+            raise ValueError(f"{name} must be [O, B, rows, ...] with src's row size")
+    _expect(pos, (B, n), "pos")
+    _raise(lib.archer_scatter_rows(
+        O, B, n, ctypes.c_size_t(row), _ptr(src, None, "src"), _ptr(pos, torch.int64, "pos"),
+        _ptr(dst0, None, "dst0"), dst0.shape[2], int(dst0_row0), _ptr(dst1, None, "dst1"),
+        0 if dst1 is None else dst1.shape[2], int(dst1_row0), _stream(stream)))
 
 
 def archer_cache_rewrite(shape: archer_shape, k_src, v_src, k_dst, v_dst, refresh_flags=None, stream=None):

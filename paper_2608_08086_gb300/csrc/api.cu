@@ -225,6 +225,23 @@ int archer_decoder_update(int batch, int resp_len, float tau_accept, float tau_r
                                changed, static_cast<cudaStream_t>(stream));
 }
 
+int archer_scatter_rows(int n_outer, int batch, int n, size_t row_bytes, const void* src, const int64_t* pos,
+                        void* dst0, int dst0_rows, int dst0_row0, void* dst1, int dst1_rows, int dst1_row0,
+                        void* stream) {
+  if (n_outer < 0 || batch < 0 || n < 0 || dst0_rows < 0 || dst0_row0 < 0 || dst1_rows < 0 || dst1_row0 < 0) {
+    set_error("negative size");
+    return ARCHER_ERR_ARG;
+  }
+  if (static_cast<long long>(n_outer) * batch * n == 0) return ARCHER_OK;
+  if (row_bytes % 16 != 0 || row_bytes / 16 > 0x7FFFFFFF) { set_error("row_bytes must be a multiple of 16"); return ARCHER_ERR_ARG; }
+  if (static_cast<long long>(n_outer) * batch * n > 0x7FFFFFFFll) { set_error("too many rows"); return ARCHER_ERR_UNSUPPORTED; }
+  int st;
+  if ((st = check_ptrs("src, pos, dst0", {src, pos, dst0}))) return st;
+  if (dst1 && (st = check_ptrs("dst1", {dst1}))) return st;
+  return scatter_rows_launch(n_outer, batch, n, row_bytes, src, pos, dst0, dst0_rows, dst0_row0, dst1, dst1_rows,
+                             dst1_row0, static_cast<cudaStream_t>(stream));
+}
+
 int archer_check_device(void* stream) {
   cudaError_t e = cudaStreamSynchronize(static_cast<cudaStream_t>(stream));
   if (e != cudaSuccess) return cuda_status(e, "cudaStreamSynchronize");

@@ -60,6 +60,9 @@ int decoder_update_launch(int B, int G, float tau_accept, float tau_remask, int3
                           const float* max_prob, const int32_t* top1, const float* cur_prob, int32_t* g,
                           uint8_t* changed, cudaStream_t stream);
 
+int scatter_rows_launch(int n_outer, int batch, int n, size_t row_bytes, const void* src, const int64_t* pos,
+                        void* dst0, int rows0, int row00, void* dst1, int rows1, int row01, cudaStream_t stream);
+
 int should_refresh_launch(int B, int G, const int32_t* g_cur, int32_t* g_anchor, int32_t* age,
                           int K, int max_age, int update_anchor, int32_t* dist, uint8_t* flag,
                           cudaStream_t stream);

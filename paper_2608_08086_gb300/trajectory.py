@@ -233,22 +233,22 @@ class DeviceTrajectory:
             self.g_host[np.arange(B)[:, None], pos] = new
             pos_d = torch.from_numpy(pos).to(self.device)
             self.g[bidx, pos_d] = torch.from_numpy(new).to(self.device)
-            for layer in range(self.L):
-                rows = synth.traj_redraw_rows(self.wl, self.seed, t, layer)
-                q, k, v = (_dev_bits(rows[c], self.device) for c in ("q", "k", "v"))
-                self.q_resp[layer][bidx, pos_d] = q
-                self.q_all[layer][bidx, P + pos_d] = q
-                self.k_resp[layer][bidx, pos_d] = k
-                self.v_resp[layer][bidx, pos_d] = v
+            rows = [synth.traj_redraw_rows(self.wl, self.seed, t, layer) for layer in range(self.L)]
+            q, k, v = (torch.stack([_dev_bits(r[c], self.device) for r in rows]) for c in ("q", "k", "v"))
         else:
             pos_d, new_d = self.plan[(t - 1) % len(self.plan)]
             self.g[bidx, pos_d] = new_d
             slot = (t - 1) % self.pool_steps
             q, k, v = self.pool["q"][slot], self.pool["k"][slot], self.pool["v"][slot]
-            self.q_resp[:, bidx, pos_d] = q
-            self.q_all[:, bidx, P + pos_d] = q
-            self.k_resp[:, bidx, pos_d] = k
-            self.v_resp[:, bidx, pos_d] = v
+        self._scatter(q, k, v, pos_d)
+
+    def _scatter(self, q, k, v, pos_d):
+        # new rows of the redrawn positions into every layer's tensors: Q into the
+        # cached step's and the refresh pass's query tensors, K and V into the
+        # response K/V (one native scatter launch each)
+        A.archer_scatter_rows(q, pos_d, self.q_resp, 0, self.q_all, self.P)
+        A.archer_scatter_rows(k, pos_d, self.k_resp)
+        A.archer_scatter_rows(v, pos_d, self.v_resp)
 
     def _stage_fresh_prompt(self, t):
         # Fresh prompt Q/K/V for a refresh (the model's prompt states under g_t).

@@ -104,3 +104,15 @@ def test_decoder_update_arguments_rejected(lib):
     assert f(2, 4, 0.9, 0.05, -1, None, p, p, p, p, None) == -1
     assert f(2, 4, float("nan"), 0.05, -1, p, p, p, p, p, None) == -1
     assert f(0, 4, 0.9, 0.05, -1, None, None, None, None, None, None) == 0
+
+
+def test_scatter_rows_arguments_rejected(lib):
+    f = lib.archer_scatter_rows
+    f.argtypes = [ctypes.c_int] * 3 + [ctypes.c_size_t] + [ctypes.c_void_p] * 3 + [ctypes.c_int] * 2 + [
+        ctypes.c_void_p] + [ctypes.c_int] * 2 + [ctypes.c_void_p]
+    p = ctypes.c_void_p(0x10000)
+    assert f(1, 1, 1, 24, p, p, p, 4, 0, None, 0, 0, None) == -1          # row_bytes % 16
+    assert f(1, 1, 1, 32, None, p, p, 4, 0, None, 0, 0, None) == -1       # NULL src
+    assert f(1, 1, 1, 32, p, p, ctypes.c_void_p(0x10008), 4, 0, None, 0, 0, None) == -1   # misaligned
+    assert f(-1, 1, 1, 32, p, p, p, 4, 0, None, 0, 0, None) == -1
+    assert f(0, 1, 1, 32, None, None, None, 0, 0, None, 0, 0, None) == 0   # nothing to do

@@ -329,3 +329,25 @@ def test_should_refresh_bit_exact(A, K, max_age):
         np.testing.assert_array_equal(flag.cpu().numpy(), rf)
         np.testing.assert_array_equal(dga.cpu().numpy(), rga)
         np.testing.assert_array_equal(dage.cpu().numpy(), rage)
+
+
+def test_scatter_rows_bit_exact(A):
+    # staging of new response rows: both destinations of a query row, and
+    # positions outside the destination skipped
+    g = torch.Generator(device="cuda").manual_seed(7)
+    L_, B, n, G, P, H, D = 3, 2, 5, 20, 7, 3, 64
+    src = torch.randn(L_, B, n, H, D, device="cuda", generator=g).to(torch.bfloat16)
+    pos = torch.tensor([[0, 3, 19, 7, 11], [2, 5, -1, 20, 1]], dtype=torch.int64, device="cuda")
+    d0 = torch.randn(L_, B, G, H, D, device="cuda", generator=g).to(torch.bfloat16)
+    d1 = torch.randn(L_, B, P + G, H, D, device="cuda", generator=g).to(torch.bfloat16)
+    e0, e1 = d0.clone(), d1.clone()
+    for b in range(B):
+        for r in range(n):
+            p = int(pos[b, r])
+            if 0 <= p < G:
+                e0[:, b, p] = src[:, b, r]
+                e1[:, b, P + p] = src[:, b, r]
+    A.archer_scatter_rows(src, pos, d0, 0, d1, P)
+    torch.cuda.synchronize()
+    assert torch.equal(d0.view(torch.int16), e0.view(torch.int16))
+    assert torch.equal(d1.view(torch.int16), e1.view(torch.int16))
