@@ -155,6 +155,7 @@ decode_scores_kernel(const T* __restrict__ logits, int64_t row_stride, int vocab
                      float* __restrict__ cur_prob, Partial* __restrict__ parts, int aligned) {
   constexpr int E = Vec<T>::kElems;              // elements per 16-byte word
   constexpr int dtype = sizeof(T) == 2 ? ARCHER_DTYPE_BF16 : ARCHER_DTYPE_F32;
+  asm volatile("griddepcontrol.launch_dependents;");   // the merge may be scheduled (it waits for this grid)
   __shared__ Smem sm;
   const int row = blockIdx.x / chunks;
   const int chunk = blockIdx.x - row * chunks;
@@ -278,6 +279,7 @@ decode_scores_bulk_kernel(const T* __restrict__ logits, int64_t row_stride, int 
   constexpr int E = Vec<T>::kElems;
   constexpr int dtype = sizeof(T) == 2 ? ARCHER_DTYPE_BF16 : ARCHER_DTYPE_F32;
   constexpr int kChunkElems = kWordsPerChunk * E;
+  asm volatile("griddepcontrol.launch_dependents;");   // the merge may be scheduled (it waits for this grid)
   extern __shared__ __align__(128) uint4 stage[];
   __shared__ Smem sm;
   __shared__ __align__(8) uint64_t full_bar;
@@ -392,8 +394,9 @@ decode_scores_bulk_kernel(const T* __restrict__ logits, int64_t row_stride, int 
   }
 }
 
-// One warp per row merges the row's chunk partials (launched after the chunk
-// kernel on the same stream).
+// One warp per row merges the row's chunk partials.  Launched as a programmatic
+// dependent of the chunk kernel on the same stream: it is scheduled while the
+// chunk grid's last wave runs and waits for that grid on the device.
 template <typename T>
 __global__ void __launch_bounds__(256)
 decode_scores_combine_kernel(const T* __restrict__ logits, int64_t row_stride, int vocab, int chunks, int rows,
@@ -401,6 +404,7 @@ decode_scores_combine_kernel(const T* __restrict__ logits, int64_t row_stride, i
                              float* __restrict__ max_prob, int32_t* __restrict__ top1, float* __restrict__ margin,
                              float* __restrict__ cur_prob, const Partial* __restrict__ parts) {
   constexpr int dtype = sizeof(T) == 2 ? ARCHER_DTYPE_BF16 : ARCHER_DTYPE_F32;
+  asm volatile("griddepcontrol.wait;" ::: "memory");
   const int row = blockIdx.x * 8 + (threadIdx.x >> 5);
   const int l = threadIdx.x & 31;
   if (row >= rows) return;
@@ -428,6 +432,23 @@ decode_scores_combine_kernel(const T* __restrict__ logits, int64_t row_stride, i
   if (l == 0)
     write_row(row, M, S, T2, I, logits + row * row_stride, dtype, vocab, mask_state, cur_tokens, max_prob, top1,
               margin, cur_prob);
+}
+
+template <typename T>
+cudaError_t launch_combine(unsigned grid, const T* logits, int64_t row_stride, int vocab, int chunks, int rows,
+                           const uint8_t* mask_state, const int32_t* cur_tokens, float* max_prob, int32_t* top1,
+                           float* margin, float* cur_prob, const Partial* parts, cudaStream_t stream) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(grid);
+  cfg.blockDim = dim3(256);
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, decode_scores_combine_kernel<T>, logits, row_stride, vocab, chunks, rows,
+                            mask_state, cur_tokens, max_prob, top1, margin, cur_prob, parts);
 }
 
 int chunks_for(int vocab, int dtype) {
@@ -476,14 +497,14 @@ int decode_scores_launch(int rows, int vocab, int dtype, const void* logits, int
           static_cast<const float*>(logits), row_stride, vocab, chunks, mask_state, cur_tokens, max_prob, top1,
           margin, cur_prob, parts, device_error_word());
     if (chunks > 1) {
-      if (dtype == ARCHER_DTYPE_BF16)
-        decode_scores_combine_kernel<__nv_bfloat16><<<combine_grid, 256, 0, stream>>>(
-            static_cast<const __nv_bfloat16*>(logits), row_stride, vocab, chunks, rows, mask_state, cur_tokens,
-            max_prob, top1, margin, cur_prob, parts);
-      else
-        decode_scores_combine_kernel<float><<<combine_grid, 256, 0, stream>>>(
-            static_cast<const float*>(logits), row_stride, vocab, chunks, rows, mask_state, cur_tokens, max_prob,
-            top1, margin, cur_prob, parts);
+      cudaError_t e = cudaGetLastError();
+      if (e == cudaSuccess)
+        e = dtype == ARCHER_DTYPE_BF16
+                ? launch_combine(combine_grid, static_cast<const __nv_bfloat16*>(logits), row_stride, vocab, chunks,
+                                 rows, mask_state, cur_tokens, max_prob, top1, margin, cur_prob, parts, stream)
+                : launch_combine(combine_grid, static_cast<const float*>(logits), row_stride, vocab, chunks, rows,
+                                 mask_state, cur_tokens, max_prob, top1, margin, cur_prob, parts, stream);
+      return cuda_status(e, "decode_scores launch");
     }
     return cuda_status(cudaGetLastError(), "decode_scores launch");
   }
@@ -491,18 +512,20 @@ int decode_scores_launch(int rows, int vocab, int dtype, const void* logits, int
     decode_scores_kernel<__nv_bfloat16><<<(unsigned)grid, kThreads, 0, stream>>>(
         static_cast<const __nv_bfloat16*>(logits), row_stride, vocab, chunks, mask_state, cur_tokens, max_prob, top1,
         margin, cur_prob, parts, aligned);
-    if (chunks > 1)
-      decode_scores_combine_kernel<__nv_bfloat16><<<combine_grid, 256, 0, stream>>>(
-          static_cast<const __nv_bfloat16*>(logits), row_stride, vocab, chunks, rows, mask_state, cur_tokens,
-          max_prob, top1, margin, cur_prob, parts);
+    if (chunks > 1 && cudaPeekAtLastError() == cudaSuccess)
+      return cuda_status(launch_combine(combine_grid, static_cast<const __nv_bfloat16*>(logits), row_stride, vocab,
+                                        chunks, rows, mask_state, cur_tokens, max_prob, top1, margin, cur_prob, parts,
+                                        stream),
+                         "decode_scores launch");
   } else {
     decode_scores_kernel<float><<<(unsigned)grid, kThreads, 0, stream>>>(
         static_cast<const float*>(logits), row_stride, vocab, chunks, mask_state, cur_tokens, max_prob, top1, margin,
         cur_prob, parts, aligned);
-    if (chunks > 1)
-      decode_scores_combine_kernel<float><<<combine_grid, 256, 0, stream>>>(
-          static_cast<const float*>(logits), row_stride, vocab, chunks, rows, mask_state, cur_tokens, max_prob, top1,
-          margin, cur_prob, parts);
+    if (chunks > 1 && cudaPeekAtLastError() == cudaSuccess)
+      return cuda_status(launch_combine(combine_grid, static_cast<const float*>(logits), row_stride, vocab, chunks,
+                                        rows, mask_state, cur_tokens, max_prob, top1, margin, cur_prob, parts,
+                                        stream),
+                         "decode_scores launch");
   }
   return cuda_status(cudaGetLastError(), "decode_scores launch");
 }
