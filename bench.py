@@ -153,18 +153,27 @@ class ClockSampler:
 
 # ---------------------------------------------------------------------------- timing helpers
 
-def barrier(dist_on):
+def barrier(dist_on, device="cuda"):
     if dist_on:
         torch.distributed.barrier()
-    torch.cuda.synchronize()
+    if device == "cuda":
+        torch.cuda.synchronize()
 
 
-def max_over_ranks(x: float, dist_on: bool) -> float:
+def max_over_ranks(x: float, dist_on: bool, device="cuda") -> float:
+    """The slowest rank's time: the job's time (replicas run in lock-step
+    between barriers)."""
     if not dist_on:
         return x
-    t = torch.tensor([x], dtype=torch.float64, device="cuda")
+    t = torch.tensor([x], dtype=torch.float64, device=device)
     torch.distributed.all_reduce(t, op=torch.distributed.ReduceOp.MAX)
     return float(t.item())
+
+
+def whole_job_rate(world: int, steps: int, ms: float) -> float:
+    """Steps per second of the whole job: every rank (one replica per GPU)
+    completes `steps` steps in the slowest rank's `ms`."""
+    return world * steps / (ms / 1e3)
 
 
 def run_arm(wl, mode, steps, warmup, dist_on, time_attention=False, seed=0):
@@ -607,7 +616,7 @@ def main():
     arm = run_arm(wl, "graph", args.steps, args.warmup, dist_on)
     clk = clocks.stop()
     ms = max_over_ranks(arm["ms"], dist_on)
-    value = world * args.steps / (ms / 1e3)
+    value = whole_job_rate(world, args.steps, ms)
     n_ref = arm["refresh_steps"]
     del arm
     torch.cuda.empty_cache()
@@ -616,7 +625,7 @@ def main():
     # durations of the roofline
     arm = run_arm(wl, "archer", args.steps, args.warmup, dist_on, time_attention=True)
     tr = arm["traj"]
-    host_value = world * args.steps / (max_over_ranks(arm["ms"], dist_on) / 1e3)
+    host_value = whole_job_rate(world, args.steps, max_over_ranks(arm["ms"], dist_on))
     ks = kernel_stats(tr)
     L = tr.L
     # per step: 3 row scatters + rule + refresh condition + L attention + scoring (2)
@@ -648,7 +657,7 @@ def main():
     # ---- the eager arm: refresh every step (one graph per step, like the Archer arm)
     eager = run_arm(wl, "eager-graph", args.eager_steps, 3, dist_on)
     eager_ms = max_over_ranks(eager["ms"], dist_on)
-    eager_value = world * args.eager_steps / (eager_ms / 1e3)
+    eager_value = whole_job_rate(world, args.eager_steps, eager_ms)
     del eager
     torch.cuda.empty_cache()
 
@@ -657,7 +666,7 @@ def main():
     if not args.no_e2e:
         e = run_e2e(wl, args.steps, args.warmup, dist_on)
         e_ms = max_over_ranks(e["ms"], dist_on)
-        e2e = {"value": world * args.steps / (e_ms / 1e3), "unit": "steps/s",
+        e2e = {"value": whole_job_rate(world, args.steps, e_ms), "unit": "steps/s",
                "h2d_bytes_per_step": e["h2d_bytes_per_step"], "d2h_bytes_per_step": e["d2h_bytes_per_step"]}
 
     # ---- a second trajectory workload (32 layers, B 8, P 1024, G 512, rule K=65 / age 8)
@@ -666,15 +675,15 @@ def main():
         wl2 = synth.WORKLOADS["traj32"]
         n2 = min(args.steps, 30)
         a2 = run_arm(wl2, "graph", n2, 3, dist_on)
-        v2 = world * n2 / (max_over_ranks(a2["ms"], dist_on) / 1e3)
+        v2 = whole_job_rate(world, n2, max_over_ranks(a2["ms"], dist_on))
         r2 = a2["refresh_steps"]
         del a2
         h2 = run_arm(wl2, "archer", n2, 3, dist_on, time_attention=True)
         ks2 = kernel_stats(h2["traj"])
-        vh2 = world * n2 / (max_over_ranks(h2["ms"], dist_on) / 1e3)
+        vh2 = whole_job_rate(world, n2, max_over_ranks(h2["ms"], dist_on))
         t2 = h2["traj"]
         e2 = run_arm(wl2, "eager-graph", args.eager_steps, 3, dist_on)
-        ve2 = world * args.eager_steps / (max_over_ranks(e2["ms"], dist_on) / 1e3)
+        ve2 = whole_job_rate(world, args.eager_steps, max_over_ranks(e2["ms"], dist_on))
         fl2 = 4.0 * t2.B * t2.Hq * t2.G * t2.N * t2.D
         secondary = {"workload": wl2.name, "steps_per_s": v2, "host_driven_steps_per_s": vh2,
                      "eager_steps_per_s": ve2, "speedup_vs_refresh_every_step": v2 / ve2, "refresh_steps": r2,
