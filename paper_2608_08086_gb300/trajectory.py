@@ -338,6 +338,35 @@ class DeviceTrajectory:
             rec["g"] = self.g.cpu().numpy()
         return rec
 
+    # ------------------------------------------------------------ checkpoint
+    _STATE = ("q_all", "q_resp", "k_resp", "v_resp", "k_new", "v_new", "k_cache", "v_cache", "g", "g_anchor", "age",
+              "dist", "flag", "refresh_count")
+    _SCORES = ("max_prob", "top1", "margin", "cur_prob", "mask_state")
+
+    def checkpoint(self) -> dict:
+        """The trajectory's state in host memory: the step, the token state
+        (g, the anchor g_r, the age), every layer's tensors -- the prompt cache
+        C_p is the state Archer carries between steps (Sec. 4.2) -- and the last
+        scores (the closed-loop decoder reads them).  restore() continues
+        bit for bit."""
+        torch.cuda.synchronize()
+        st = {"t": self.t, "n_refresh": self._n_refresh_steps, "g_host": self.g_host.copy()}
+        for name in self._STATE + self._SCORES:
+            if hasattr(self, name):
+                st[name] = getattr(self, name).detach().cpu().clone()
+        return st
+
+    def restore(self, st: dict):
+        """Loads a checkpoint() into this trajectory's (same-shaped) tensors,
+        in place: a step graph captured on them stays valid."""
+        for name in self._STATE + self._SCORES:
+            if name in st:
+                getattr(self, name).copy_(st[name])
+        self.t = st["t"]
+        self._n_refresh_steps = st["n_refresh"]
+        self.g_host = st["g_host"].copy()
+        torch.cuda.synchronize()
+
     def attention_flops(self, refresh: bool) -> float:
         """Algorithmic attention FLOPs of one step over all layers: 4 B Hq M N D
         (Q K^T and P V, 2 flops per multiply-add), M = N on refresh, G cached."""

@@ -152,3 +152,33 @@ def test_closed_loop_decoder_trajectory_matches_oracle(dev_mode):
         for k in ("max_prob", "margin", "cur_prob"):
             err = np.abs(s_got[k] - s_ref[k]) - (1e-5 + 1e-4 * np.abs(s_ref[k]))
             assert (err <= 0).all(), f"{k} at step {t}"
+
+
+@pytest.mark.parametrize("mode,decoder", [("archer", "redraw"), ("graph", "closed")])
+def test_checkpoint_restore_continues_bit_for_bit(mode, decoder):
+    # the prompt cache is the state: a trajectory stopped after 4 steps and
+    # restored into a fresh one continues exactly like the uninterrupted run
+    import dataclasses
+    from paper_2608_08086_gb300.trajectory import DeviceTrajectory
+    wl = dataclasses.replace(MIXED, steps=9) if decoder == "redraw" else _closed_workload()
+    kw = dict(seed=24, mode=mode, source="host", record=True, decoder=decoder)
+    full = DeviceTrajectory(wl, **kw)
+    full.build()
+    ref = [full.step() for _ in range(wl.steps)]
+    a = DeviceTrajectory(wl, **kw)
+    a.build()
+    for _ in range(4):
+        a.step()
+    ck = a.checkpoint()
+    del a
+    b = DeviceTrajectory(wl, **kw)
+    b.restore(ck)
+    for r in ref[4:]:
+        g = b.step()
+        assert g["t"] == r["t"]
+        np.testing.assert_array_equal(g["flag"], r["flag"])
+        np.testing.assert_array_equal(g["g"], r["g"])
+        assert torch.equal(g["out"][-1].view(torch.int16), r["out"][-1].view(torch.int16))
+        for k in r["scores"]:
+            assert torch.equal(g["scores"][k], r["scores"][k])
+    assert b.n_refresh_steps == full.n_refresh_steps
