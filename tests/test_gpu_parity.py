@@ -209,6 +209,43 @@ def test_attention_full_size_gqa_long_sampled(A):
     assert torch.equal(kc, d["k_prompt"]) and torch.equal(vc, d["v_prompt"])
 
 
+@pytest.mark.parametrize("case,full", [
+    ((1, 512, 256, 32, 32, 128), True),     # the LLaDA-shaped layer, every row (latency-bound grid)
+    ((1, 2048, 256, 32, 32, 128), False),   # prompt-sweep end: the cached step splits its 18 key tiles
+    ((8, 1024, 512, 32, 32, 128), False),   # the 32-layer trajectory's layer (3.4 waves of CTAs)
+])
+def test_attention_config_shapes(A, case, full):
+    B, P, G, Hq, Hkv, D = case
+    sh = synth.AttnShape(B, P, G, Hq, Hkv, D)
+    d = synth.device_attn_inputs(sh, "cuda", seed=11)
+    N, scale = P + G, 1.0 / math.sqrt(D)
+    shape = A.make_shape(B, P, G, Hq, Hkv, D)
+    out_s = torch.empty(B, G, Hq, D, dtype=torch.bfloat16, device="cuda")
+    q_resp = d["q_all"][:, P:].contiguous()
+    A.archer_attn_step(shape, q_resp, d["k_cache"], d["v_cache"], d["k_resp"], d["v_resp"], out_s)
+    out_r = torch.empty(B, N, Hq, D, dtype=torch.bfloat16, device="cuda")
+    A.archer_prompt_refresh(shape, d["q_all"], d["k_prompt"], d["v_prompt"], d["k_resp"], d["v_resp"], out_r,
+                            None, d["k_prompt"], d["v_prompt"])
+    torch.cuda.synchronize()
+    A.archer_check_device()
+    rng = np.random.default_rng(1)
+    heads = range(Hq) if full else [0, Hq // 2, Hq - 1]
+    for b in ([0] if full else [0, B - 1]):
+        for h in heads:
+            kvh = h // (Hq // Hkv)
+            sl = (slice(b, b + 1), slice(None), slice(kvh, kvh + 1))
+            kg, vg = host_f64(d["k_resp"][sl]), host_f64(d["v_resp"][sl])
+            rows_s = np.arange(G) if full else np.unique(np.concatenate([[0, G - 1], rng.integers(0, G, 24)]))
+            ref, _ = O.attention(host_f64(q_resp[b:b + 1, rows_s, h:h + 1]), host_f64(d["k_cache"][sl]),
+                                 host_f64(d["v_cache"][sl]), kg, vg, scale)
+            assert_attn_close(host_f64(out_s[b:b + 1, rows_s, h:h + 1]), ref, f"{case} step b{b} h{h}")
+            rows_r = np.arange(N) if full else np.unique(np.concatenate([[0, P - 1, P, N - 1],
+                                                                          rng.integers(0, N, 24)]))
+            ref, _ = O.attention(host_f64(d["q_all"][b:b + 1, rows_r, h:h + 1]), host_f64(d["k_prompt"][sl]),
+                                 host_f64(d["v_prompt"][sl]), kg, vg, scale)
+            assert_attn_close(host_f64(out_r[b:b + 1, rows_r, h:h + 1]), ref, f"{case} refresh b{b} h{h}")
+
+
 # ----------------------------------------------------------------------------
 # decoder scoring
 # ----------------------------------------------------------------------------
