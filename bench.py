@@ -440,20 +440,20 @@ def run_e2e(wl, steps, warmup, dist_on, seed=0):
     layer_ready = [torch.cuda.Event() for _ in range(L)]
     tr.layer_ready = layer_ready
 
-    # the prompt rows of q_all are strided ([B, N, Hq, D]): upload into a
-    # contiguous staging buffer at full link speed, then scatter on the device
-    d_q_prompt = torch.empty_like(h_q_prompt, device=tr.device)
-
     def stage_fresh(t):
         # Per-layer uploads on their own stream: layer l's refresh waits only for
         # its own prompt Q/K/V, so later layers' copies overlap earlier layers' work.
+        # The prompt rows of q_all ([B, N, Hq, D]) are contiguous per sequence:
+        # one host-to-device copy each, done by the copy engine (a strided
+        # destination would need a device kernel, competing with the attention
+        # for SMs).
         here = torch.cuda.Event()
         here.record()
         with torch.cuda.stream(fresh_stream):
             fresh_stream.wait_event(here)
             for layer in range(L):
-                d_q_prompt.copy_(h_q_prompt, non_blocking=True)
-                tr.q_all[layer][:, :P].copy_(d_q_prompt)
+                for b in range(B):
+                    tr.q_all[layer][b, :P].copy_(h_q_prompt[b], non_blocking=True)
                 tr.k_new[layer].copy_(h_k_new, non_blocking=True)
                 tr.v_new[layer].copy_(h_v_new, non_blocking=True)
                 layer_ready[layer].record(fresh_stream)
