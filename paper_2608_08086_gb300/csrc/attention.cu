@@ -77,6 +77,7 @@ struct AttnParams {
   // and writes its unnormalised O, running max and row sum to the workspace
   // instead of out; attn_combine_kernel merges the splits.
   int n_split, tiles_per_split;
+  int tiles_per_cta;          // query tiles per CTA: 2 (ping-pong), or 1 for grids far below the SM count
   float* ws_o;                // [n_split, B, Hq, M, D] fp32
   float2* ws_ml;              // [n_split, B, Hq, M] (max in log2 units, row sum)
 };
@@ -180,9 +181,9 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
   // of this grid is resident; it still waits for this grid's completion.
   asm volatile("griddepcontrol.launch_dependents;");
   const bool refresh = p.flags ? (p.flags[b] != 0) : (p.default_refresh != 0);
-  const int q0 = (refresh ? p.q_begin_refresh : p.q_begin_cached) + tp * 2 * kBM;
+  const int q0 = (refresh ? p.q_begin_refresh : p.q_begin_cached) + tp * p.tiles_per_cta * kBM;
   if (q0 >= p.M) return;  // uniform over the CTA, before any barrier or TMEM use
-  const bool has_b = q0 + kBM < p.M;
+  const bool has_b = p.tiles_per_cta == 2 && q0 + kBM < p.M;
 
   const int kvh = h / (p.Hq / p.Hkv);
   const int n_p = (p.P + kBN - 1) / kBN;
@@ -503,7 +504,7 @@ int sm_count() {
 }
 
 struct SplitPlan {
-  int n_split = 1, per = 0;
+  int tiles_per_cta = 2, n_split = 1, per = 0;
   size_t bytes = 0;
 };
 
@@ -512,12 +513,19 @@ struct SplitPlan {
 // splits as whole grids fit on the SMs, none empty.  Measured on the GB300
 // (B 1, 32 heads, G 256): P 2048 (T 18) 38 -> 26 us, P 1024 (T 10) 26 -> 23 us,
 // while T <= 6 gains nothing over a CTA's fixed start-up and the merge.
+//
+// Before that, a grid of two-tile CTAs that would still fill at most half the
+// SMs runs one query tile per CTA instead: twice the CTAs, each key step
+// shorter (one tile's MMAs and softmax), for latency-bound launches.
 SplitPlan split_plan(int B, int P, int G, int Hq, int D, int rows, int M) {
   SplitPlan sp;
   const int T = (P + kBN - 1) / kBN + (G + kBN - 1) / kBN;
   sp.per = T;
-  const long long ctas = static_cast<long long>((rows + 2 * kBM - 1) / (2 * kBM)) * Hq * B;
   const int sms = sm_count();
+  const long long pairs = static_cast<long long>((rows + 2 * kBM - 1) / (2 * kBM)) * Hq * B;
+  if (sms > 0 && rows > kBM && 2 * pairs <= sms) sp.tiles_per_cta = 1;
+  const int rows_per_cta = sp.tiles_per_cta * kBM;
+  const long long ctas = static_cast<long long>((rows + rows_per_cta - 1) / rows_per_cta) * Hq * B;
   if (ctas <= 0 || sms <= 0 || ctas >= sms || T < kMinSplitTiles) return sp;
   int s = static_cast<int>(std::min<long long>(std::min(T, kMaxSplit), sms / ctas));
   if (s < 2) return sp;
@@ -600,6 +608,7 @@ int launch_d(const AttnCall& c, cudaStream_t stream) {
   // Query tiles needed by the longest query range (a refreshed sequence's).
   const int rows = c.M - (c.flags || c.default_refresh ? c.q_begin_refresh : c.q_begin_cached);
   SplitPlan sp = split_plan(c.B, c.P, c.G, c.Hq, D, rows, c.M);
+  prm.tiles_per_cta = sp.tiles_per_cta;
   if (sp.n_split > 1 && (!c.ws || c.ws_bytes < sp.bytes || (reinterpret_cast<uintptr_t>(c.ws) & 15u))) {
     sp.n_split = 1;                                 // no (usable) workspace: one CTA per tile pair
     sp.per = (c.P + kBN - 1) / kBN + (c.G + kBN - 1) / kBN;
@@ -613,7 +622,8 @@ int launch_d(const AttnCall& c, cudaStream_t stream) {
     prm.ws_ml = reinterpret_cast<float2*>(static_cast<char*>(c.ws) +
                                           static_cast<size_t>(sp.n_split) * c.B * c.Hq * c.M * D * 4);
   }
-  const dim3 grid(((rows + 2 * kBM - 1) / (2 * kBM)) * sp.n_split, c.Hq, c.B);
+  const int rows_per_cta = sp.tiles_per_cta * kBM;
+  const dim3 grid(((rows + rows_per_cta - 1) / rows_per_cta) * sp.n_split, c.Hq, c.B);
   attn_fwd_kernel<D><<<grid, kThreads, L::kSmemBytes, stream>>>(mq, mkr, mvr, mkc, mvc, mkg, mvg, prm);
   int st = cuda_status(cudaGetLastError(), "attention launch");
   if (st || sp.n_split == 1) return st;
