@@ -285,14 +285,21 @@ typedef struct archer_step_graph archer_step_graph;
 
 /* Validates desc, captures and instantiates the graph (host work, done once;
  * the capture runs on a private stream and launches nothing).  *out receives
- * the handle.  Calls no cudaMalloc; the graph's own objects are the CUDA
- * runtime's. */
+ * the handle (NULL on failure).  Calls no cudaMalloc; the graph's own objects
+ * are the CUDA runtime's.  Errors: ARCHER_ERR_ARG for a NULL desc/out, no
+ * layers, batch < 1, missing rule buffers or scoring outputs, and whatever
+ * status the captured calls return for their arguments (the same checks as
+ * when called directly); ARCHER_ERR_CUDA if capture or instantiation fails.
+ * Nothing is left half-built. */
 int archer_step_graph_create(const archer_step_desc* desc, archer_step_graph** out);
 
-/* Launches one step on `stream`. */
+/* Launches one step on `stream` (asynchronous; ARCHER_ERR_ARG for a NULL
+ * graph, ARCHER_ERR_CUDA if the launch fails).  Device-side wait timeouts
+ * inside the step surface through archer_check_device, as for direct calls. */
 int archer_step_graph_launch(archer_step_graph* graph, void* stream);
 
-/* Frees the graph (after its last launch has completed). */
+/* Frees the graph; call it after the graph's last launch has completed.
+ * NULL is a no-op. */
 int archer_step_graph_destroy(archer_step_graph* graph);
 
 /* Reads and clears the device-side error word that kernels set when a

@@ -269,6 +269,6 @@ const char* archer_status_string(int status) {
 
 const char* archer_last_error(void) { return g_last_error; }
 
-int archer_version(void) { return 100; }
+int archer_version(void) { return 200; }
 
 }  // extern "C"

@@ -36,7 +36,7 @@ def test_status_strings_and_version(lib):
     lib.archer_status_string.restype = ctypes.c_char_p
     assert lib.archer_status_string(0) == b"ok"
     assert lib.archer_status_string(-4) == b"device wait timed out"
-    assert lib.archer_version() >= 100
+    assert lib.archer_version() >= 200      # 0.2.0: step graph, decoder stand-in, row scatter
 
 
 class Shape(ctypes.Structure):
