@@ -177,8 +177,12 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
   extern __shared__ uint8_t smem_raw[];
 
   const int tp = blockIdx.x / p.n_split, split = blockIdx.x % p.n_split, h = blockIdx.y, b = blockIdx.z;
-  // Lets a programmatic dependent (the split merge) be scheduled once every CTA
-  // of this grid is resident; it still waits for this grid's completion.
+  // Launched as a programmatic dependent of the stream's previous kernel: wait
+  // for it before reading anything it may have written (flags, Q/K/V).
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+  // Lets a programmatic dependent (the split merge, the next layer) be
+  // scheduled once every CTA of this grid is resident; it still waits for
+  // this grid's completion.
   asm volatile("griddepcontrol.launch_dependents;");
   const bool refresh = p.flags ? (p.flags[b] != 0) : (p.default_refresh != 0);
   const int q0 = (refresh ? p.q_begin_refresh : p.q_begin_cached) + tp * p.tiles_per_cta * kBM;
@@ -624,8 +628,20 @@ int launch_d(const AttnCall& c, cudaStream_t stream) {
   }
   const int rows_per_cta = sp.tiles_per_cta * kBM;
   const dim3 grid(((rows + rows_per_cta - 1) / rows_per_cta) * sp.n_split, c.Hq, c.B);
-  attn_fwd_kernel<D><<<grid, kThreads, L::kSmemBytes, stream>>>(mq, mkr, mvr, mkc, mvc, mkg, mvg, prm);
-  int st = cuda_status(cudaGetLastError(), "attention launch");
+  // A programmatic dependent launch: its launch latency overlaps the previous
+  // kernel on the stream, which every CTA waits for before its first read.
+  cudaLaunchConfig_t lc = {};
+  lc.gridDim = grid;
+  lc.blockDim = dim3(kThreads);
+  lc.dynamicSmemBytes = L::kSmemBytes;
+  lc.stream = stream;
+  cudaLaunchAttribute la[1];
+  la[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  la[0].val.programmaticStreamSerializationAllowed = 1;
+  lc.attrs = la;
+  lc.numAttrs = 1;
+  int st = cuda_status(cudaLaunchKernelEx(&lc, attn_fwd_kernel<D>, mq, mkr, mvr, mkc, mvc, mkg, mvg, prm),
+                       "attention launch");
   if (st || sp.n_split == 1) return st;
   // The merge is a programmatic dependent launch: it is scheduled while the
   // attention grid still runs and waits for it on the device.
