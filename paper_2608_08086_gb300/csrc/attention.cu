@@ -78,6 +78,11 @@ struct AttnParams {
   // instead of out; attn_combine_kernel merges the splits.
   int n_split, tiles_per_split;
   int tiles_per_cta;          // query tiles per CTA: 2 (ping-pong), or 1 for grids far below the SM count
+  // Flat grid: CTA x < n_unit_ctas is unit x, units numbered (tile pair x
+  // split) fastest, then head, then sequence; the CTAs after them each take one
+  // tile of the last n_tail_pairs tile pairs (a nearly empty last wave of pairs
+  // becomes one wave of single tiles).
+  int B, tiles_x, n_unit_ctas;
   float* ws_o;                // [n_split, B, Hq, M, D] fp32
   float2* ws_ml;              // [n_split, B, Hq, M] (max in log2 units, row sum)
 };
@@ -176,7 +181,15 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
   using L = Layout<D>;
   extern __shared__ uint8_t smem_raw[];
 
-  const int tp = blockIdx.x / p.n_split, split = blockIdx.x % p.n_split, h = blockIdx.y, b = blockIdx.z;
+  int unit = blockIdx.x, tile_off = 0;
+  const bool tail_single = unit >= p.n_unit_ctas;
+  if (tail_single) {                      // one tile of a tail pair (no splits here)
+    tile_off = (unit - p.n_unit_ctas) & 1;
+    unit = p.n_unit_ctas + ((unit - p.n_unit_ctas) >> 1);
+  }
+  const int tpx = unit % p.tiles_x;
+  const int h = (unit / p.tiles_x) % p.Hq, b = unit / (p.tiles_x * p.Hq);
+  const int tp = tpx / p.n_split, split = tpx % p.n_split;
   // Launched as a programmatic dependent of the stream's previous kernel: wait
   // for it before reading anything it may have written (flags, Q/K/V).
   asm volatile("griddepcontrol.wait;" ::: "memory");
@@ -185,9 +198,9 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
   // this grid's completion.
   asm volatile("griddepcontrol.launch_dependents;");
   const bool refresh = p.flags ? (p.flags[b] != 0) : (p.default_refresh != 0);
-  const int q0 = (refresh ? p.q_begin_refresh : p.q_begin_cached) + tp * p.tiles_per_cta * kBM;
+  const int q0 = (refresh ? p.q_begin_refresh : p.q_begin_cached) + (tp * p.tiles_per_cta + tile_off) * kBM;
   if (q0 >= p.M) return;  // uniform over the CTA, before any barrier or TMEM use
-  const bool has_b = p.tiles_per_cta == 2 && q0 + kBM < p.M;
+  const bool has_b = !tail_single && p.tiles_per_cta == 2 && q0 + kBM < p.M;
 
   const int kvh = h / (p.Hq / p.Hkv);
   const int n_p = (p.P + kBN - 1) / kBN;
@@ -401,7 +414,7 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
       const int q = q0 + t * kBM + r;
       const bool live = ok && q < p.M;
       if (partial) {
-        const size_t row = ((static_cast<size_t>(split) * gridDim.z + b) * p.Hq + h) * p.M + q;
+        const size_t row = ((static_cast<size_t>(split) * p.B + b) * p.Hq + h) * p.M + q;
         float* orow_ws = p.ws_o + row * D;
 #pragma unroll
         for (int c0 = 0; c0 < D; c0 += 32) {
@@ -627,7 +640,23 @@ int launch_d(const AttnCall& c, cudaStream_t stream) {
                                           static_cast<size_t>(sp.n_split) * c.B * c.Hq * c.M * D * 4);
   }
   const int rows_per_cta = sp.tiles_per_cta * kBM;
-  const dim3 grid(((rows + rows_per_cta - 1) / rows_per_cta) * sp.n_split, c.Hq, c.B);
+  prm.B = c.B;
+  prm.tiles_x = ((rows + rows_per_cta - 1) / rows_per_cta) * sp.n_split;
+  const long long units = static_cast<long long>(prm.tiles_x) * c.Hq * c.B;
+  if (units > 0x3FFFFFFFll) {
+    set_error("too many attention work units (%lld)", units);
+    return ARCHER_ERR_UNSUPPORTED;
+  }
+  // A last wave of tile pairs at most half full runs as one wave of single
+  // tiles instead: each of its SMs then finishes in about 0.7 of a pair's time.
+  int tail = 0;
+  const int sms = sm_count();
+  if (sp.n_split == 1 && sp.tiles_per_cta == 2 && sms > 0 && units > sms) {
+    const int r = static_cast<int>(units % sms);
+    if (r > 0 && 2 * r <= sms) tail = r;
+  }
+  prm.n_unit_ctas = static_cast<int>(units) - tail;
+  const dim3 grid(static_cast<unsigned>(units + tail));
   // A programmatic dependent launch: its launch latency overlaps the previous
   // kernel on the stream, which every CTA waits for before its first read.
   cudaLaunchConfig_t lc = {};
