@@ -57,7 +57,7 @@ MEASURED_TRAFFIC = {
     # (kernel, workload): DRAM bytes read + written per launch from one ncu capture
     # (dram__bytes_read.sum + dram__bytes_write.sum), valid only while the kernel's
     # sources hash to sha16 (sha256 over the listed files, first 16 hex digits).
-    ("attn_step", "gqa_long"): {"bytes": 251403264, "sha16": "b241ce393ebfa410",
+    ("attn_step", "gqa_long"): {"bytes": 251477248, "sha16": "cf43873b1e6b4194",
                                 "sources": ["attention.cu", "archer_device.cuh", "tmem_ldst.cuh"]},
     ("scores", "gqa_long"): {"bytes": 2496017152, "sha16": "b7e42a718e51535f",
                              "sources": ["decode_scores.cu", "archer_device.cuh"]},
