@@ -270,47 +270,19 @@ __device__ __forceinline__ void bulk_load(uint32_t dst, const void* src, uint32_
                : "memory");
 }
 
-template <typename T>
-__global__ void __launch_bounds__(kThreads, 6)
-decode_scores_bulk_kernel(const T* __restrict__ logits, int64_t row_stride, int vocab, int chunks,
-                          const uint8_t* __restrict__ mask_state, const int32_t* __restrict__ cur_tokens,
-                          float* __restrict__ max_prob, int32_t* __restrict__ top1, float* __restrict__ margin,
-                          float* __restrict__ cur_prob, Partial* __restrict__ parts, int* __restrict__ err) {
+// Pass A (top-2 of the chunk, block-wide) and pass B (sum of exponentials
+// against the chunk max, lowest index of the max) over one staged chunk.
+// kFull: the chunk holds kWordsPerChunk whole 16-byte words (every chunk of
+// a row but possibly its last), so no word needs a bounds check.
+template <typename T, bool kFull>
+__device__ __forceinline__ void chunk_pass(const uint4* __restrict__ stage, int bulk_words, const T* zrow,
+                                           int64_t e0c, int n_el, Smem& sm, float& m_blk, float& t2_blk,
+                                           float& sum, int& idx) {
   constexpr int E = Vec<T>::kElems;
   constexpr int dtype = sizeof(T) == 2 ? ARCHER_DTYPE_BF16 : ARCHER_DTYPE_F32;
-  constexpr int kChunkElems = kWordsPerChunk * E;
-  asm volatile("griddepcontrol.launch_dependents;");   // the merge may be scheduled (it waits for this grid)
-  extern __shared__ __align__(128) uint4 stage[];
-  __shared__ Smem sm;
-  __shared__ __align__(8) uint64_t full_bar;
-  __shared__ int abort_flag;
-  const int row = blockIdx.x / chunks;
-  const int chunk = blockIdx.x - row * chunks;
-  const T* zrow = logits + row * row_stride;
-  const int64_t e0c = static_cast<int64_t>(chunk) * kChunkElems;
-  const int n_el = static_cast<int>(min(static_cast<int64_t>(kChunkElems), static_cast<int64_t>(vocab) - e0c));
-  const uint32_t bytes = (static_cast<uint32_t>(n_el) * sizeof(T)) & ~15u;
-  const int bulk_words = static_cast<int>(bytes / 16);
-  const uint32_t bar = smem_u32(&full_bar);
-  if (threadIdx.x == 0) {
-    abort_flag = 0;
-    mbar_init(bar, 1);
-    mbar_fence_init();
-    if (bytes > 0) {
-      mbar_arrive_expect_tx(bar, bytes);
-      bulk_load(smem_u32(stage), zrow + e0c, bytes, bar);
-    } else {
-      mbar_arrive(bar);
-    }
-  }
-  __syncthreads();
-  // An expired wait is reported through the error word; the CTA then reads
-  // stale shared memory (in bounds) rather than leaving early.
-  mbar_wait(bar, 0, &abort_flag, err);
-
   auto word = [&](int u) -> uint4 {
     const int wi = u * kThreads + threadIdx.x;
-    if (wi < bulk_words) return stage[wi];
+    if (kFull || wi < bulk_words) return stage[wi];
     float v[E];
 #pragma unroll
     for (int e = 0; e < E; ++e) {
@@ -357,20 +329,27 @@ decode_scores_bulk_kernel(const T* __restrict__ logits, int64_t row_stride, int 
     }
   }
   const float my_t1 = t1;
-  float m_blk = t1, t2_blk = t2;
+  m_blk = t1;
+  t2_blk = t2;
   block_top2(m_blk, t2_blk, sm);
 
   // pass B: one ex2 per logit against the chunk max; lowest index of the max
   const float neg_m = (m_blk == -INFINITY) ? 0.f : -m_blk * kLog2e;
-  float sum = 0.f;
+  // packed fp32 pairs: one FMA and one add instruction per two logits
+  const float2 l2e = make_float2(kLog2e, kLog2e), nm = make_float2(neg_m, neg_m);
+  float2 acc[2] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
 #pragma unroll
   for (int u = 0; u < kUnroll; ++u) {
     float v[E];
     unpack(word(u), v, (T*)nullptr);
 #pragma unroll
-    for (int e = 0; e < E; ++e) sum += ex2_approx(fmaf(v[e], kLog2e, neg_m));
+    for (int e = 0; e < E; e += 2) {
+      const float2 y = ffma2(make_float2(v[e], v[e + 1]), l2e, nm);
+      acc[(e >> 1) & 1] = fadd2(acc[(e >> 1) & 1], make_float2(ex2_approx(y.x), ex2_approx(y.y)));
+    }
   }
-  int idx = INT_MAX;
+  sum = (acc[0].x + acc[0].y) + (acc[1].x + acc[1].y);
+  idx = INT_MAX;
   if (my_t1 == m_blk) {
     for (int u = 0; u < kUnroll && idx == INT_MAX; ++u) {
       float v[E];
@@ -381,6 +360,52 @@ decode_scores_bulk_kernel(const T* __restrict__ logits, int64_t row_stride, int 
         if (v[e] == m_blk) idx = static_cast<int>(el0 + e);
     }
   }
+}
+
+template <typename T>
+__global__ void __launch_bounds__(kThreads, 6)
+decode_scores_bulk_kernel(const T* __restrict__ logits, int64_t row_stride, int vocab, int chunks,
+                          const uint8_t* __restrict__ mask_state, const int32_t* __restrict__ cur_tokens,
+                          float* __restrict__ max_prob, int32_t* __restrict__ top1, float* __restrict__ margin,
+                          float* __restrict__ cur_prob, Partial* __restrict__ parts, int* __restrict__ err) {
+  constexpr int E = Vec<T>::kElems;
+  constexpr int dtype = sizeof(T) == 2 ? ARCHER_DTYPE_BF16 : ARCHER_DTYPE_F32;
+  constexpr int kChunkElems = kWordsPerChunk * E;
+  asm volatile("griddepcontrol.launch_dependents;");   // the merge may be scheduled (it waits for this grid)
+  extern __shared__ __align__(128) uint4 stage[];
+  __shared__ Smem sm;
+  __shared__ __align__(8) uint64_t full_bar;
+  __shared__ int abort_flag;
+  const int row = blockIdx.x / chunks;
+  const int chunk = blockIdx.x - row * chunks;
+  const T* zrow = logits + row * row_stride;
+  const int64_t e0c = static_cast<int64_t>(chunk) * kChunkElems;
+  const int n_el = static_cast<int>(min(static_cast<int64_t>(kChunkElems), static_cast<int64_t>(vocab) - e0c));
+  const uint32_t bytes = (static_cast<uint32_t>(n_el) * sizeof(T)) & ~15u;
+  const int bulk_words = static_cast<int>(bytes / 16);
+  const uint32_t bar = smem_u32(&full_bar);
+  if (threadIdx.x == 0) {
+    abort_flag = 0;
+    mbar_init(bar, 1);
+    mbar_fence_init();
+    if (bytes > 0) {
+      mbar_arrive_expect_tx(bar, bytes);
+      bulk_load(smem_u32(stage), zrow + e0c, bytes, bar);
+    } else {
+      mbar_arrive(bar);
+    }
+  }
+  __syncthreads();
+  // An expired wait is reported through the error word; the CTA then reads
+  // stale shared memory (in bounds) rather than leaving early.
+  mbar_wait(bar, 0, &abort_flag, err);
+
+  float m_blk, t2_blk, sum;
+  int idx;
+  if (bulk_words == kWordsPerChunk)
+    chunk_pass<T, true>(stage, bulk_words, zrow, e0c, n_el, sm, m_blk, t2_blk, sum, idx);
+  else
+    chunk_pass<T, false>(stage, bulk_words, zrow, e0c, n_el, sm, m_blk, t2_blk, sum, idx);
   block_sum_minidx(sum, idx, sm);
   if (threadIdx.x == 0) {
     if (chunks == 1) {
