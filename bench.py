@@ -57,9 +57,9 @@ MEASURED_TRAFFIC = {
     # (kernel, workload): DRAM bytes read + written per launch from one ncu capture
     # (dram__bytes_read.sum + dram__bytes_write.sum), valid only while the kernel's
     # sources hash to sha16 (sha256 over the listed files, first 16 hex digits).
-    ("attn_step", "gqa_long"): {"bytes": 251477248, "sha16": "cf43873b1e6b4194",
+    ("attn_step", "gqa_long"): {"bytes": 251062016, "sha16": "24fb2ced993c7c50",
                                 "sources": ["attention.cu", "archer_device.cuh", "tmem_ldst.cuh"]},
-    ("scores", "gqa_long"): {"bytes": 2496017152, "sha16": "b7e42a718e51535f",
+    ("scores", "gqa_long"): {"bytes": 2496203264, "sha16": "78100384823fbe81",
                              "sources": ["decode_scores.cu", "archer_device.cuh"]},
 }
 
