@@ -282,7 +282,8 @@ __device__ __forceinline__ void chunk_pass(const uint4* __restrict__ stage, int 
   constexpr int dtype = sizeof(T) == 2 ? ARCHER_DTYPE_BF16 : ARCHER_DTYPE_F32;
   auto word = [&](int u) -> uint4 {
     const int wi = u * kThreads + threadIdx.x;
-    if (kFull || wi < bulk_words) return stage[wi];
+    if constexpr (kFull) return stage[wi];
+    if (wi < bulk_words) return stage[wi];
     float v[E];
 #pragma unroll
     for (int e = 0; e < E; ++e) {
