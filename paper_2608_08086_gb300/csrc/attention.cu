@@ -110,6 +110,9 @@ struct Layout {
 // .sync.aligned, so all 32 lanes must take the same path).
 __device__ __forceinline__ bool warp_wait(uint32_t bar, uint32_t parity, volatile int* abort,
                                           int* err, long long limit) {
+  // The first poll reads no clock: an already complete phase costs one
+  // try_wait and one vote.
+  if (__all_sync(0xffffffffu, mbar_try_wait(bar, parity))) return true;
   const long long t0 = clock64();
   while (true) {
     const bool done = mbar_try_wait(bar, parity);
