@@ -99,12 +99,23 @@ struct Layout {
   static constexpr int kBars = 1 + 2 * kSlots + 4;
   static constexpr uint32_t kOffHolder = kOffBar + 8 * kBars;
   static constexpr uint32_t kOffAbort = kOffHolder + 4;
-  static constexpr uint32_t kUsed = kOffAbort + 4;
+  static constexpr uint32_t kOffDrain = kOffAbort + 4;        // abort path: the MMA warp's MMAs done
+  static constexpr uint32_t kUsed = kOffDrain + 8;
   // + 1 KB to align the base to 1024 B; at least 120 KB so that one CTA
   // holds an SM (the CTA allocates all 512 TMEM columns).
   static constexpr uint32_t kSmemBytes = (kUsed + 1024 > 120 * 1024) ? kUsed + 1024 : 120 * 1024;
   static_assert(kUsed + 1024 <= 232448, "shared memory budget");
 };
+
+// Warp-uniform wait bounded by the clock alone (the abort flag is already
+// set when it runs): lets in-flight MMAs and copies land before the CTA frees
+// TMEM or exits.  Returns whether the phase completed.
+__device__ __forceinline__ bool drain_wait(uint32_t bar, uint32_t parity, long long limit) {
+  const long long t0 = clock64();
+  while (!__all_sync(0xffffffffu, mbar_try_wait(bar, parity)))
+    if (__any_sync(0xffffffffu, clock64() - t0 > limit)) return false;
+  return true;
+}
 
 // Warp-uniform bounded wait for the softmax warps (tcgen05.ld/st are
 // .sync.aligned, so all 32 lanes must take the same path).
@@ -204,6 +215,7 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
   const uint32_t bar_empty = bar_full + 8 * L::kSlots;          // + 8 * slot
   const uint32_t bar_s_full = bar_empty + 8 * L::kSlots;        // + 8 * tile (A = 0, B = 1)
   const uint32_t bar_p_full = bar_s_full + 16;                  // + 8 * tile: both halves of P written
+  const uint32_t bar_drain = base + L::kOffDrain;
   uint32_t* holder = reinterpret_cast<uint32_t*>(gbase + L::kOffHolder);
   volatile int* abort = reinterpret_cast<volatile int*>(gbase + L::kOffAbort);
 
@@ -231,6 +243,8 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
   const uint32_t tmem = *holder;
 
   const bool lane0 = (threadIdx.x & 31) == 0;
+  int last_pair = -1;          // producer: the last pair whose loads were issued
+  bool mma_done = false;       // MMA warp: every MMA issued and committed to the S barriers
   if (warp == kWarpProducer) {
     // ------------------------------------------------------------ producer
     // The whole warp runs the loop and waits (warp-uniform); lane 0 issues.
@@ -245,7 +259,8 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
     }
     __syncwarp();
     // pair u = (V_{u-1}, K_u) into pair slot u & 1: [V tile | K tile]
-    for (int u = 0; u <= T; ++u) {
+    int u = 0;
+    for (; u <= T; ++u) {
       const int slot = u & 1, use = u >> 1;
       if (use > 0 && !warp_wait(bar_empty + 8 * slot, (use - 1) & 1, abort, p.err, p.wait_limit)) break;
       if (lane0) {
@@ -263,6 +278,7 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
       }
       __syncwarp();
     }
+    last_pair = u - 1;         // the loop breaks before issuing pair u
   } else if (warp == kWarpMma) {
     // ------------------------------------------------------------ MMA issuer
     // The whole warp runs the loop and waits (warp-uniform); lane 0 issues
@@ -303,7 +319,8 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
       }
       __syncwarp();
     }
-    for (int j = 0; ok && j < T; ++j) {
+    int j = 0;
+    for (; ok && j < T; ++j) {
       const bool more = j + 1 < T;
       const int u = j + 1;                    // pair (V_j, K_{j+1})
       if (!warp_wait(bar_full + 8 * (u & 1), phase_of(u), abort, p.err, p.wait_limit)) break;
@@ -322,6 +339,7 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
       if (lane0) umma_commit(bar_empty + 8 * (u & 1));
       __syncwarp();
     }
+    mma_done = ok && j == T;
   } else {
     // ------------------------------------------------------------ softmax
     const int t = (warp - kWarpSoftmax0) >> 2;                    // 0 = tile A, 1 = tile B
@@ -437,10 +455,27 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
 
   tc_fence_before();
   __syncthreads();
+  // After an expired wait no role may leave work in flight: the MMA warp
+  // waits for its MMAs before TMEM is freed, and the producer for the loads
+  // it issued before the CTA's shared memory is released (both bounded).
+  const bool aborted = *abort != 0;
   if (warp == kWarpMma) {
+    if (aborted || !mma_done) {
+      if (lane0) {
+        mbar_init(bar_drain, 1);
+        mbar_fence_init();
+        umma_commit(bar_drain);
+      }
+      __syncwarp();
+      drain_wait(bar_drain, 0, p.wait_limit);
+    }
     __syncwarp();
     tc_fence_after();
     tmem_dealloc(tmem, kTmemCols);
+  } else if (warp == kWarpProducer && aborted) {
+    drain_wait(bar_q_full, 0, p.wait_limit);
+    for (int u = max(0, last_pair - 1); u <= last_pair; ++u)
+      drain_wait(bar_full + 8 * (u & 1), static_cast<uint32_t>(u >> 1) & 1u, p.wait_limit);
   }
 }
 
