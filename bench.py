@@ -239,6 +239,30 @@ def kernel_only(args, wl):
     return 0
 
 
+def _time_graph(fn, runs):
+    """Mean duration in us of fn's launches replayed back to back from one CUDA
+    graph of `runs` launches: the device-side cost, free of the host's launch
+    rate (which bounds plain back-to-back launches of layers this small)."""
+    g = torch.cuda.CUDAGraph()
+    side = torch.cuda.Stream()
+    side.wait_stream(torch.cuda.current_stream())
+    with torch.cuda.stream(side):
+        fn()
+    torch.cuda.current_stream().wait_stream(side)
+    with torch.cuda.graph(g):
+        for _ in range(runs):
+            fn()
+    g.replay()
+    torch.cuda.synchronize()
+    s, e = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    s.record()
+    g.replay()
+    e.record()
+    e.synchronize()
+    del g
+    return s.elapsed_time(e) * 1e3 / runs
+
+
 def _time_launches(fn, runs, flush=None):
     """Median (cold: L2 flushed before each launch) and mean back-to-back
     duration in us of fn's launches, CUDA events on the current stream."""
@@ -281,9 +305,10 @@ def _attn_pair(sh, dev, runs, flush):
     res = {}
     for name, fn, M in (("step", step, G), ("refresh", refresh, N)):
         cold, b2b = _time_launches(fn, runs, flush)
+        gr = _time_graph(fn, runs)
         fl = 4.0 * B * Hq * M * N * D
-        res[name] = {"cold_us": cold, "b2b_us": b2b, "gflop": fl / 1e9, "tflops_cold": fl / cold / 1e6,
-                     "tflops_b2b": fl / b2b / 1e6}
+        res[name] = {"cold_us": cold, "b2b_us": b2b, "graph_us": gr, "gflop": fl / 1e9, "tflops_cold": fl / cold / 1e6,
+                     "tflops_b2b": fl / b2b / 1e6, "tflops_graph": fl / gr / 1e6}
     A.archer_check_device()
     res["refresh_over_step"] = res["refresh"]["cold_us"] / res["step"]["cold_us"]
     res["ideal_ratio_N_over_G"] = N / G
@@ -295,7 +320,8 @@ def sweep(args):
     layer (B1, 32 = 32 heads, D128, P512, G256), decoder scoring on
     [4 x 256 x 126464] bf16, and the prompt-length sweep G = 256,
     P = 128 ... 2048 with LLaDA heads (cached step vs refresh of one layer).
-    "cold" launches follow a 256 MB L2-flushing write; "b2b" is back to back."""
+    "cold" launches follow a 256 MB L2-flushing write; "b2b" is back to back
+    from the host; "graph" is back to back from one captured CUDA graph."""
     from paper_2608_08086_gb300 import archer as A
     dev = torch.device("cuda")
     pk, pk_kind = peaks()
@@ -315,9 +341,11 @@ def sweep(args):
     for _ in range(3):
         fn()
     cold, b2b = _time_launches(fn, runs, flush)
+    gr = _time_graph(fn, runs)
     nbytes = rows * wl.vocab * 2
     print(json.dumps({"sweep": "scoring", "rows": rows, "vocab": wl.vocab, "bytes": nbytes, "cold_us": cold,
-                      "b2b_us": b2b, "gbs_cold": nbytes / cold / 1e3, "frac_cold": nbytes / cold / 1e3 / pk["hbm_gbs"],
+                      "b2b_us": b2b, "graph_us": gr, "gbs_cold": nbytes / cold / 1e3,
+                      "frac_cold": nbytes / cold / 1e3 / pk["hbm_gbs"],
                       "peak_gbs": pk["hbm_gbs"], "peak_kind": pk_kind}), flush=True)
     for P in (128, 256, 512, 1024, 2048):
         sh = synth.AttnShape(1, P, 256, 32, 32, 128)

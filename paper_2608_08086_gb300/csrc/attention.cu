@@ -36,6 +36,15 @@
 //              more issue slots than the shorter rows saved.)
 // TMEM (512 columns): S_A [0,128) S_B [128,256) O_A [256,256+D) O_B [384,384+D).
 // Every hand-off is an mbarrier; every wait is bounded (archer_device.cuh).
+//
+// Launches whose grid would fill at most half the SMs take one query tile per
+// CTA and run the one-tile instantiation (kSingle): the free TMEM columns
+// double-buffer S (S(j) in [128 (j % 2), +128), O in [256, 256+D)), so the MMA
+// warp computes S(j+2) while the softmax works on S(j+1) and the key step
+// costs the longer of one tile's MMAs and one tile's softmax rather than their
+// sum.  With one Q tile in shared memory there is room for three K/V pair
+// slots.  A barrier "O done" (completed after each P V) lets the softmax
+// rescale O only once P V of the previous tile has finished.
 
 #include <cmath>
 #include <cstdio>
@@ -87,20 +96,23 @@ struct AttnParams {
   float2* ws_ml;              // [n_split, B, Hq, M] (max in log2 units, row sum)
 };
 
-template <int D>
+// kSingle: the one-tile kernel (one Q tile, three pair slots, S double
+// buffered in TMEM, one more barrier for "O holds P V up to tile j").
+template <int D, bool kSingle = false>
 struct Layout {
   static constexpr int kChunks = D / 64;                    // 128-byte column chunks
   static constexpr uint32_t kTile = kChunks * kChunkBytes;  // one 128-row tile of D bf16
-  static constexpr int kSlots = 2;                          // pair slots: [V tile | K tile]
-  static constexpr uint32_t kOffQ = 0;                      // Q_A, Q_B
-  static constexpr uint32_t kOffKV = kOffQ + 2 * kTile;
+  static constexpr int kSlots = kSingle ? 3 : 2;            // pair slots: [V tile | K tile]
+  static constexpr uint32_t kOffQ = 0;                      // Q_A, Q_B (Q only when kSingle)
+  static constexpr uint32_t kOffKV = kOffQ + (kSingle ? 1 : 2) * kTile;
   static constexpr uint32_t kOffBar = kOffKV + kSlots * 2 * kTile;
   // q_full, full[slots], empty[slots], s_full[2], p_full[2]
   static constexpr int kBars = 1 + 2 * kSlots + 4;
   static constexpr uint32_t kOffHolder = kOffBar + 8 * kBars;
   static constexpr uint32_t kOffAbort = kOffHolder + 4;
   static constexpr uint32_t kOffDrain = kOffAbort + 4;        // abort path: the MMA warp's MMAs done
-  static constexpr uint32_t kUsed = kOffDrain + 8;
+  static constexpr uint32_t kOffODone = kOffDrain + 8;        // kSingle: P V up to tile j complete
+  static constexpr uint32_t kUsed = kOffDrain + (kSingle ? 16 : 8);
   // + 1 KB to align the base to 1024 B; at least 120 KB so that one CTA
   // holds an SM (the CTA allocates all 512 TMEM columns).
   static constexpr uint32_t kSmemBytes = (kUsed + 1024 > 120 * 1024) ? kUsed + 1024 : 120 * 1024;
@@ -165,14 +177,17 @@ __device__ __forceinline__ void load_scores128(uint32_t taddr, int valid, float 
   }
 }
 
-template <int D>
+template <int D, bool kSingle>
 __global__ void __launch_bounds__(kThreads, 1)
 attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
                 const __grid_constant__ CUtensorMap tmKpR, const __grid_constant__ CUtensorMap tmVpR,
                 const __grid_constant__ CUtensorMap tmKpC, const __grid_constant__ CUtensorMap tmVpC,
                 const __grid_constant__ CUtensorMap tmKg, const __grid_constant__ CUtensorMap tmVg,
                 const AttnParams p) {
-  using L = Layout<D>;
+  using L = Layout<D, kSingle>;
+  // pair u lives in slot u mod kSlots, that slot's use u div kSlots
+  auto slot_of = [](int u) { return L::kSlots == 2 ? (u & 1) : (u % L::kSlots); };
+  auto use_of = [](int u) { return L::kSlots == 2 ? (u >> 1) : (u / L::kSlots); };
   extern __shared__ uint8_t smem_raw[];
 
   int unit = blockIdx.x, tile_off = 0;
@@ -216,11 +231,34 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
   const uint32_t bar_s_full = bar_empty + 8 * L::kSlots;        // + 8 * tile (A = 0, B = 1)
   const uint32_t bar_p_full = bar_s_full + 16;                  // + 8 * tile: both halves of P written
   const uint32_t bar_drain = base + L::kOffDrain;
+  const uint32_t bar_o_done = base + L::kOffODone;               // kSingle only
   uint32_t* holder = reinterpret_cast<uint32_t*>(gbase + L::kOffHolder);
   volatile int* abort = reinterpret_cast<volatile int*>(gbase + L::kOffAbort);
 
   const int warp = threadIdx.x >> 5;
-  if (threadIdx.x == 0) {
+  const bool lane0 = (threadIdx.x & 31) == 0;
+  const CUtensorMap* mKp = refresh ? &tmKpR : &tmKpC;
+  const CUtensorMap* mVp = refresh ? &tmVpR : &tmVpC;
+  // Producer lane 0: pair u = (V_{u-1}, K_u) into its pair slot, [V tile | K tile].
+  auto issue_pair = [&](int u) {
+    const int slot = slot_of(u);
+    const bool has_v = u >= 1, has_k = u < T;
+    mbar_arrive_expect_tx(bar_full + 8 * slot, (has_v && has_k ? 2 : 1) * L::kTile);
+    for (int part = has_v ? 0 : 1; part < (has_k ? 2 : 1); ++part) {
+      const int j = j0 + (part == 0 ? u - 1 : u);             // global key tile
+      const bool in_prompt = j < n_p;
+      const int row = in_prompt ? j * kBN : (j - n_p) * kBN;
+      const CUtensorMap* map = in_prompt ? (part == 0 ? mVp : mKp) : (part == 0 ? &tmVg : &tmKg);
+      const uint32_t dst = sKV + (2 * slot + part) * L::kTile;
+      for (int c = 0; c < L::kChunks; ++c)
+        tma_load_4d(dst + c * kChunkBytes, map, bar_full + 8 * slot, c * 64, kvh, row, b);
+    }
+  };
+  // The producer's lane 0 sets up the barriers and issues the Q tiles and
+  // the pairs whose slots start free before the CTA-wide barrier, so those
+  // loads overlap the TMEM allocation and the barrier itself.
+  const int u_pre = min(L::kSlots, T + 1);
+  if (warp == kWarpProducer && lane0) {
     mbar_init(bar_q_full, 1);
     for (int s = 0; s < L::kSlots; ++s) {
       mbar_init(bar_full + 8 * s, 1);
@@ -230,8 +268,15 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
       mbar_init(bar_s_full + 8 * i, 1);
       mbar_init(bar_p_full + 8 * i, kBM);
     }
+    if constexpr (kSingle) mbar_init(bar_o_done, 1);
     *abort = 0;
     mbar_fence_init();
+    tma_prefetch_map(&tmQ);
+    mbar_arrive_expect_tx(bar_q_full, has_b ? 2 * L::kTile : L::kTile);
+    for (int t = 0; t < (has_b ? 2 : 1); ++t)
+      for (int c = 0; c < L::kChunks; ++c)
+        tma_load_4d(sQ + t * L::kTile + c * kChunkBytes, &tmQ, bar_q_full, c * 64, h, q0 + t * kBM, b);
+    for (int u = 0; u < u_pre; ++u) issue_pair(u);
   }
   if (warp == kWarpMma) {
     tmem_alloc(smem_u32(holder), kTmemCols);
@@ -242,40 +287,16 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
   tc_fence_after();
   const uint32_t tmem = *holder;
 
-  const bool lane0 = (threadIdx.x & 31) == 0;
   int last_pair = -1;          // producer: the last pair whose loads were issued
   bool mma_done = false;       // MMA warp: every MMA issued and committed to the S barriers
   if (warp == kWarpProducer) {
     // ------------------------------------------------------------ producer
     // The whole warp runs the loop and waits (warp-uniform); lane 0 issues.
-    const CUtensorMap* mKp = refresh ? &tmKpR : &tmKpC;
-    const CUtensorMap* mVp = refresh ? &tmVpR : &tmVpC;
-    if (lane0) {
-      tma_prefetch_map(&tmQ);
-      mbar_arrive_expect_tx(bar_q_full, has_b ? 2 * L::kTile : L::kTile);
-      for (int t = 0; t < (has_b ? 2 : 1); ++t)
-        for (int c = 0; c < L::kChunks; ++c)
-          tma_load_4d(sQ + t * L::kTile + c * kChunkBytes, &tmQ, bar_q_full, c * 64, h, q0 + t * kBM, b);
-    }
-    __syncwarp();
-    // pair u = (V_{u-1}, K_u) into pair slot u & 1: [V tile | K tile]
-    int u = 0;
+    int u = u_pre;
     for (; u <= T; ++u) {
-      const int slot = u & 1, use = u >> 1;
+      const int slot = slot_of(u), use = use_of(u);
       if (use > 0 && !warp_wait(bar_empty + 8 * slot, (use - 1) & 1, abort, p.err, p.wait_limit)) break;
-      if (lane0) {
-        const bool has_v = u >= 1, has_k = u < T;
-        mbar_arrive_expect_tx(bar_full + 8 * slot, (has_v && has_k ? 2 : 1) * L::kTile);
-        for (int part = has_v ? 0 : 1; part < (has_k ? 2 : 1); ++part) {
-          const int j = j0 + (part == 0 ? u - 1 : u);             // global key tile
-          const bool in_prompt = j < n_p;
-          const int row = in_prompt ? j * kBN : (j - n_p) * kBN;
-          const CUtensorMap* map = in_prompt ? (part == 0 ? mVp : mKp) : (part == 0 ? &tmVg : &tmKg);
-          const uint32_t dst = sKV + (2 * slot + part) * L::kTile;
-          for (int c = 0; c < L::kChunks; ++c)
-            tma_load_4d(dst + c * kChunkBytes, map, bar_full + 8 * slot, c * 64, kvh, row, b);
-        }
-      }
+      if (lane0) issue_pair(u);
       __syncwarp();
     }
     last_pair = u - 1;         // the loop breaks before issuing pair u
@@ -303,43 +324,117 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
         umma_ts(tmem + col_o(t), tmem + col_s(t) + 64 * (kk >> 2) + (kk & 3) * 8,
                 sdesc_sw128(v_tile + kk * 2048, kChunkBytes, 1024), idesc_pv, (acc || kk > 0) ? 1u : 0u);
     };
-    auto v_tile_of = [&](int u) { return sKV + 2 * (u & 1) * L::kTile; };
-    auto k_tile_of = [&](int u) { return sKV + (2 * (u & 1) + 1) * L::kTile; };
-    auto phase_of = [](int u) { return static_cast<uint32_t>(u >> 1) & 1u; };
-    bool ok = warp_wait(bar_q_full, 0, abort, p.err, p.wait_limit) &&
-              warp_wait(bar_full, phase_of(0), abort, p.err, p.wait_limit);
-    if (ok) {
-      if (lane0) {
-        tc_fence_after();
-        for (int t = 0; t < n_tiles; ++t) {
-          issue_qk(t, k_tile_of(0));
-          umma_commit(bar_s_full + 8 * t);
+    auto v_tile_of = [&](int u) { return sKV + 2 * slot_of(u) * L::kTile; };
+    auto k_tile_of = [&](int u) { return sKV + (2 * slot_of(u) + 1) * L::kTile; };
+    auto phase_of = [&](int u) { return static_cast<uint32_t>(use_of(u)) & 1u; };
+    if constexpr (kSingle) {
+      // One query tile, S double buffered: S(j) in buffer j & 1 (columns
+      // col_s(j & 1), P(j) written over it), O in col_o(0).  Per key tile j:
+      // wait P(j); O += P(j) V_j; commit "O done" (its j-th completion) and
+      // free pair j + 1; then S(j + 2) = Q K_{j+2}^T into the buffer P(j) came
+      // from (issue order: P V reads P(j) first).  The softmax of tile j + 1
+      // runs meanwhile on the other buffer, so the key step is the longer of
+      // one tile's MMAs and one tile's softmax instead of their sum.
+      auto issue_qk1 = [&](int bf, uint32_t k_tile) {
+#pragma unroll
+        for (int kk = 0; kk < D / 16; ++kk) {
+          const uint32_t off = (kk >> 2) * kChunkBytes + (kk & 3) * 32;
+          umma_ss(tmem + col_s(bf), sdesc_sw128(sQ + off, 16, 1024), sdesc_sw128(k_tile + off, 16, 1024),
+                  idesc_qk, kk > 0 ? 1u : 0u);
         }
-        umma_commit(bar_empty);               // pair 0 (K_0) read
-      }
-      __syncwarp();
-    }
-    int j = 0;
-    for (; ok && j < T; ++j) {
-      const bool more = j + 1 < T;
-      const int u = j + 1;                    // pair (V_j, K_{j+1})
-      if (!warp_wait(bar_full + 8 * (u & 1), phase_of(u), abort, p.err, p.wait_limit)) break;
-      for (int t = 0; t < n_tiles; ++t) {
-        if (!warp_wait(bar_p_full + 8 * t, j & 1, abort, p.err, p.wait_limit)) { ok = false; break; }
-        if (p.debug_skip_last_pv && !more) { ok = false; break; }   // the softmax's final wait must expire
+      };
+      auto issue_pv1 = [&](int bf, uint32_t v_tile, bool acc) {
+#pragma unroll
+        for (int kk = 0; kk < 8; ++kk)
+          umma_ts(tmem + col_o(0), tmem + col_s(bf) + 64 * (kk >> 2) + (kk & 3) * 8,
+                  sdesc_sw128(v_tile + kk * 2048, kChunkBytes, 1024), idesc_pv, (acc || kk > 0) ? 1u : 0u);
+      };
+      // pairs 0 (K_0) and 1 (V_0, K_1): S(0) and S(1)
+      bool ok = warp_wait(bar_q_full, 0, abort, p.err, p.wait_limit) &&
+                warp_wait(bar_full, phase_of(0), abort, p.err, p.wait_limit);
+      if (ok) {
         if (lane0) {
           tc_fence_after();
-          issue_pv(t, v_tile_of(u), j > 0);
-          if (more) issue_qk(t, k_tile_of(u));
-          umma_commit(bar_s_full + 8 * t);   // S_t(j+1) ready -- or, after the last tile, O_t final
+          issue_qk1(0, k_tile_of(0));
+          umma_commit(bar_s_full);
+          umma_commit(bar_empty + 8 * slot_of(0));
+        }
+        __syncwarp();
+        ok = warp_wait(bar_full + 8 * slot_of(1), phase_of(1), abort, p.err, p.wait_limit);
+      }
+      if (ok && T > 1) {
+        if (lane0) {
+          tc_fence_after();
+          issue_qk1(1, k_tile_of(1));
+          umma_commit(bar_s_full + 8);
         }
         __syncwarp();
       }
-      if (!ok) break;
-      if (lane0) umma_commit(bar_empty + 8 * (u & 1));
-      __syncwarp();
+      int j = 0;
+      for (; ok && j < T; ++j) {
+        const int u = j + 1;                  // pair (V_j, K_{j+1})
+        const bool more2 = j + 2 < T;         // S(j + 2) to compute
+        // pair u was waited for S(j + 1), except the last pair (V_{T-1} only)
+        if (j + 1 == T && T > 1 && !warp_wait(bar_full + 8 * slot_of(u), phase_of(u), abort, p.err, p.wait_limit))
+          break;
+        if (!warp_wait(bar_p_full + 8 * (j & 1), static_cast<uint32_t>(j >> 1) & 1u, abort, p.err, p.wait_limit)) {
+          ok = false;
+          break;
+        }
+        if (p.debug_skip_last_pv && j + 1 == T) { ok = false; break; }   // the softmax's final wait must expire
+        if (more2 && !warp_wait(bar_full + 8 * slot_of(u + 1), phase_of(u + 1), abort, p.err, p.wait_limit)) {
+          ok = false;
+          break;
+        }
+        if (lane0) {
+          tc_fence_after();
+          issue_pv1(j & 1, v_tile_of(u), j > 0);
+          umma_commit(bar_o_done);
+          umma_commit(bar_empty + 8 * slot_of(u));
+          if (more2) {
+            issue_qk1(j & 1, k_tile_of(u + 1));
+            umma_commit(bar_s_full + 8 * (j & 1));
+          }
+        }
+        __syncwarp();
+      }
+      mma_done = ok && j == T;
+    } else {
+      bool ok = warp_wait(bar_q_full, 0, abort, p.err, p.wait_limit) &&
+                warp_wait(bar_full, phase_of(0), abort, p.err, p.wait_limit);
+      if (ok) {
+        if (lane0) {
+          tc_fence_after();
+          for (int t = 0; t < n_tiles; ++t) {
+            issue_qk(t, k_tile_of(0));
+            umma_commit(bar_s_full + 8 * t);
+          }
+          umma_commit(bar_empty);               // pair 0 (K_0) read
+        }
+        __syncwarp();
+      }
+      int j = 0;
+      for (; ok && j < T; ++j) {
+        const bool more = j + 1 < T;
+        const int u = j + 1;                    // pair (V_j, K_{j+1})
+        if (!warp_wait(bar_full + 8 * (u & 1), phase_of(u), abort, p.err, p.wait_limit)) break;
+        for (int t = 0; t < n_tiles; ++t) {
+          if (!warp_wait(bar_p_full + 8 * t, j & 1, abort, p.err, p.wait_limit)) { ok = false; break; }
+          if (p.debug_skip_last_pv && !more) { ok = false; break; }   // the softmax's final wait must expire
+          if (lane0) {
+            tc_fence_after();
+            issue_pv(t, v_tile_of(u), j > 0);
+            if (more) issue_qk(t, k_tile_of(u));
+            umma_commit(bar_s_full + 8 * t);   // S_t(j+1) ready -- or, after the last tile, O_t final
+          }
+          __syncwarp();
+        }
+        if (!ok) break;
+        if (lane0) umma_commit(bar_empty + 8 * (u & 1));
+        __syncwarp();
+      }
+      mma_done = ok && j == T;
     }
-    mma_done = ok && j == T;
   } else {
     // ------------------------------------------------------------ softmax
     const int t = (warp - kWarpSoftmax0) >> 2;                    // 0 = tile A, 1 = tile B
@@ -366,18 +461,25 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
       // An expired wait sets the abort flag; the warps then run on over stale
       // TMEM (in bounds) to the epilogue.
       for (int j = 0; j < T; ++j) {
-        warp_wait(bar_s, j & 1, abort, p.err, p.wait_limit);
+        // kSingle: S(j), P(j) in buffer j & 1 (its (j / 2)-th use)
+        const uint32_t bar_sj = kSingle ? bar_s_full + 8 * (j & 1) : bar_s;
+        const uint32_t bar_pj = kSingle ? bar_p_full + 8 * (j & 1) : bar_ph;
+        const uint32_t col_sj = kSingle ? col_s(j & 1) : colS;
+        warp_wait(bar_sj, kSingle ? (j >> 1) & 1 : j & 1, abort, p.err, p.wait_limit);
         tc_fence_after();
         const int jg = j0 + j;
         const int valid = jg < n_p ? min(kBN, p.P - jg * kBN) : min(kBN, p.G - (jg - n_p) * kBN);
         // The row's 128 scores are read from TMEM once and kept in registers.
         float x[128];
-        load_scores128(t_lane + colS, valid, x);
+        load_scores128(t_lane + col_sj, valid, x);
         const float tm = max128(x) * sl2;
         if (j == 0) {
           m_used = tm;
         } else if (__any_sync(0xffffffffu, tm > m_used + 8.0f)) {
-          // O holds P V up to tile j-1, complete (S(j) was announced after it).
+          // O must hold P V up to tile j-1, complete: with two tiles S(j) was
+          // announced after it; with one, wait for "O done" of tile j-1 (the
+          // barrier cannot be further ahead: P V of tile j needs this P).
+          if constexpr (kSingle) warp_wait(bar_o_done, (j - 1) & 1, abort, p.err, p.wait_limit);
           const float m_new = fmaxf(m_used, tm);
           const float a = ex2_approx(m_used - m_new);
           m_used = m_new;
@@ -402,14 +504,22 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
             acc[k & 1] = fadd2(acc[k & 1], pr);
             pk[k] = pack_bf16x2(pr.x, pr.y);
           }
-          tmem_st_16_async(t_lane + colS + 64 * (q >> 1) + 16 * (q & 1), pk);
+          tmem_st_16_async(t_lane + col_sj + 64 * (q >> 1) + 16 * (q & 1), pk);
         }
         tmem_wait_st();
         l2 = fadd2(l2, fadd2(acc[0], acc[1]));
         tc_fence_before();
-        mbar_arrive(bar_ph);
+        mbar_arrive(bar_pj);
       }
-      const bool ok = warp_wait(bar_s, T & 1, abort, p.err, p.wait_limit);
+      bool ok;
+      if constexpr (kSingle) {
+        // O final = "O done" of tile T-1; the barrier may be two phases behind
+        // (S(T-1) was issued before P V of tile T-2), so take them in order.
+        ok = (T < 2 || warp_wait(bar_o_done, (T - 2) & 1, abort, p.err, p.wait_limit)) &&
+             warp_wait(bar_o_done, (T - 1) & 1, abort, p.err, p.wait_limit);
+      } else {
+        ok = warp_wait(bar_s, T & 1, abort, p.err, p.wait_limit);
+      }
       tc_fence_after();
       const float l_sum = l2.x + l2.y;
       const int q = q0 + t * kBM + r;
@@ -474,8 +584,8 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
     tmem_dealloc(tmem, kTmemCols);
   } else if (warp == kWarpProducer && aborted) {
     drain_wait(bar_q_full, 0, p.wait_limit);
-    for (int u = max(0, last_pair - 1); u <= last_pair; ++u)
-      drain_wait(bar_full + 8 * (u & 1), static_cast<uint32_t>(u >> 1) & 1u, p.wait_limit);
+    for (int u = max(0, last_pair - (L::kSlots - 1)); u <= last_pair; ++u)
+      drain_wait(bar_full + 8 * slot_of(u), static_cast<uint32_t>(use_of(u)) & 1u, p.wait_limit);
   }
 }
 
@@ -601,13 +711,15 @@ bool make_map(CUtensorMap* map, const void* ptr, int B, int L, int H, int D) {
 
 template <int D>
 int launch_d(const AttnCall& c, cudaStream_t stream) {
-  using L = Layout<D>;
   static int configured_device = -1;
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess) return cuda_status(cudaGetLastError(), "cudaGetDevice");
   if (configured_device != dev) {
-    cudaError_t e = cudaFuncSetAttribute(attn_fwd_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                         (int)L::kSmemBytes);
+    cudaError_t e = cudaFuncSetAttribute(attn_fwd_kernel<D, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                         (int)Layout<D, false>::kSmemBytes);
+    if (e == cudaSuccess)
+      e = cudaFuncSetAttribute(attn_fwd_kernel<D, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                               (int)Layout<D, true>::kSmemBytes);
     if (e != cudaSuccess) return cuda_status(e, "cudaFuncSetAttribute(attention)");
     configured_device = dev;
   }
@@ -677,17 +789,20 @@ int launch_d(const AttnCall& c, cudaStream_t stream) {
   const dim3 grid(static_cast<unsigned>(units + tail));
   // A programmatic dependent launch: its launch latency overlaps the previous
   // kernel on the stream, which every CTA waits for before its first read.
+  // One query tile per CTA runs the one-tile kernel (S double buffered).
+  const bool single = sp.tiles_per_cta == 1;
   cudaLaunchConfig_t lc = {};
   lc.gridDim = grid;
   lc.blockDim = dim3(kThreads);
-  lc.dynamicSmemBytes = L::kSmemBytes;
+  lc.dynamicSmemBytes = single ? Layout<D, true>::kSmemBytes : Layout<D, false>::kSmemBytes;
   lc.stream = stream;
   cudaLaunchAttribute la[1];
   la[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
   la[0].val.programmaticStreamSerializationAllowed = 1;
   lc.attrs = la;
   lc.numAttrs = 1;
-  int st = cuda_status(cudaLaunchKernelEx(&lc, attn_fwd_kernel<D>, mq, mkr, mvr, mkc, mvc, mkg, mvg, prm),
+  int st = cuda_status(single ? cudaLaunchKernelEx(&lc, attn_fwd_kernel<D, true>, mq, mkr, mvr, mkc, mvc, mkg, mvg, prm)
+                              : cudaLaunchKernelEx(&lc, attn_fwd_kernel<D, false>, mq, mkr, mvr, mkc, mvc, mkg, mvg, prm),
                        "attention launch");
   if (st || sp.n_split == 1) return st;
   // The merge is a programmatic dependent launch: it is scheduled while the
