@@ -57,7 +57,7 @@ MEASURED_TRAFFIC = {
     # (kernel, workload): DRAM bytes read + written per launch from one ncu capture
     # (dram__bytes_read.sum + dram__bytes_write.sum), valid only while the kernel's
     # sources hash to sha16 (sha256 over the listed files, first 16 hex digits).
-    ("attn_step", "gqa_long"): {"bytes": 250685696, "sha16": "aabbdb2ff33c9231",
+    ("attn_step", "gqa_long"): {"bytes": 247218176, "sha16": "634525748ceb8fa5",
                                 "sources": ["attention.cu", "archer_device.cuh", "tmem_ldst.cuh"]},
     ("scores", "gqa_long"): {"bytes": 2496017920, "sha16": "f609be40559ef555",
                              "sources": ["decode_scores.cu", "archer_device.cuh"]},
@@ -597,7 +597,7 @@ def main():
     ap.add_argument("--steps", type=int, default=20)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
-    ap.add_argument("--workload", default="gqa_long", choices=["gqa_long", "traj32"])
+    ap.add_argument("--workload", default="gqa_long", choices=["gqa_long", "traj32", "llada_layer"])
     ap.add_argument("--eager-steps", type=int, default=4)
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu", action="store_true")
@@ -611,6 +611,8 @@ def main():
                     help="per-configuration measurements (LLaDA layer, scoring, prompt-length sweep)")
     args = ap.parse_args()
     args.warmup = max(args.warmup, 3)
+    if args.workload == "llada_layer" and args.kernel_only not in ("attn_step", "attn_refresh"):
+        ap.error("llada_layer is a single attention layer: use it with --kernel-only attn_step|attn_refresh")
     wl = synth.WORKLOADS[args.workload]
 
     if args.impl == "reference":
@@ -743,7 +745,7 @@ def main():
             "speedup_vs_refresh_every_step": value / eager_value,
             "eager_steps_per_s": eager_value,
             "attention": att,
-            "roofline": {"bound": "tensor", "kernel": "attn_fwd_kernel<128>", "launches": "cached step",
+            "roofline": {"bound": "tensor", "kernel": "attn_fwd_kernel<128, false>", "launches": "cached step",
                          "flops_per_launch": flops_step_launch, "achieved": achieved, "peak": peak_tf,
                          "unit": "TFLOP/s", "frac": achieved / peak_tf,
                          "traffic": measured_traffic("attn_step", wl.name),
