@@ -1,6 +1,6 @@
 """Failure detection without a GPU fault: a host-set test hook makes the
 attention kernel withhold its last P V product, so the softmax warps' bounded
-wait expires.  The kernel must leave cleanly (TMEM freed, no trap, no hang),
+wait expires (in both kernel instantiations).  The kernel must leave cleanly (TMEM freed, no trap, no hang),
 archer_check_device must report ARCHER_ERR_TIMEOUT, and the context must stay
 usable: the next call is correct."""
 import math
@@ -15,9 +15,13 @@ from paper_2608_08086_gb300 import synth
 pytestmark = pytest.mark.gpu
 
 
-def test_expired_wait_reports_timeout_and_context_survives(monkeypatch):
+# G = 64: two-tile kernel (one CTA holds the only query tile pair); G = 256:
+# the launch plan takes one tile per CTA, so the one-tile kernel (S double
+# buffered, "O done" barrier) runs its own abort path.
+@pytest.mark.parametrize("G", [64, 256], ids=["two-tile", "one-tile"])
+def test_expired_wait_reports_timeout_and_context_survives(monkeypatch, G):
     from paper_2608_08086_gb300 import archer as A
-    B, P, G, H, D = 1, 128, 64, 2, 64
+    B, P, H, D = 1, 128, 2, 64
     bits = synth.attn_inputs(synth.AttnShape(B, P, G, H, H, D), seed=9)
     d = {k: torch.from_numpy(v.view(np.int16)).view(torch.bfloat16).cuda() for k, v in bits.items()}
     shape = A.make_shape(B, P, G, H, H, D)
