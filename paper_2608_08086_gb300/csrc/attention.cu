@@ -43,8 +43,8 @@
 // warp computes S(j+2) while the softmax works on S(j+1) and the key step
 // costs the longer of one tile's MMAs and one tile's softmax rather than their
 // sum.  With one Q tile in shared memory there is room for three K/V pair
-// slots.  A barrier "O done" (completed after each P V) lets the softmax
-// rescale O only once P V of the previous tile has finished.
+// slots.  The S barrier's commit after each P V also tells the softmax when O
+// may be rescaled and, after the last one, that O is final.
 
 #include <cmath>
 #include <cstdio>
@@ -97,7 +97,7 @@ struct AttnParams {
 };
 
 // kSingle: the one-tile kernel (one Q tile, three pair slots, S double
-// buffered in TMEM, one more barrier for "O holds P V up to tile j").
+// buffered in TMEM).
 template <int D, bool kSingle = false>
 struct Layout {
   static constexpr int kChunks = D / 64;                    // 128-byte column chunks
@@ -111,8 +111,7 @@ struct Layout {
   static constexpr uint32_t kOffHolder = kOffBar + 8 * kBars;
   static constexpr uint32_t kOffAbort = kOffHolder + 4;
   static constexpr uint32_t kOffDrain = kOffAbort + 4;        // abort path: the MMA warp's MMAs done
-  static constexpr uint32_t kOffODone = kOffDrain + 8;        // kSingle: P V up to tile j complete
-  static constexpr uint32_t kUsed = kOffDrain + (kSingle ? 16 : 8);
+  static constexpr uint32_t kUsed = kOffDrain + 8;
   // + 1 KB to align the base to 1024 B; at least 120 KB so that one CTA
   // holds an SM (the CTA allocates all 512 TMEM columns).
   static constexpr uint32_t kSmemBytes = (kUsed + 1024 > 120 * 1024) ? kUsed + 1024 : 120 * 1024;
@@ -231,7 +230,6 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
   const uint32_t bar_s_full = bar_empty + 8 * L::kSlots;        // + 8 * tile (A = 0, B = 1)
   const uint32_t bar_p_full = bar_s_full + 16;                  // + 8 * tile: both halves of P written
   const uint32_t bar_drain = base + L::kOffDrain;
-  const uint32_t bar_o_done = base + L::kOffODone;               // kSingle only
   uint32_t* holder = reinterpret_cast<uint32_t*>(gbase + L::kOffHolder);
   volatile int* abort = reinterpret_cast<volatile int*>(gbase + L::kOffAbort);
 
@@ -268,7 +266,6 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
       mbar_init(bar_s_full + 8 * i, 1);
       mbar_init(bar_p_full + 8 * i, kBM);
     }
-    if constexpr (kSingle) mbar_init(bar_o_done, 1);
     *abort = 0;
     mbar_fence_init();
     tma_prefetch_map(&tmQ);
@@ -330,11 +327,13 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
     if constexpr (kSingle) {
       // One query tile, S double buffered: S(j) in buffer j & 1 (columns
       // col_s(j & 1), P(j) written over it), O in col_o(0).  Per key tile j:
-      // wait P(j); O += P(j) V_j; commit "O done" (its j-th completion) and
-      // free pair j + 1; then S(j + 2) = Q K_{j+2}^T into the buffer P(j) came
-      // from (issue order: P V reads P(j) first).  The softmax of tile j + 1
-      // runs meanwhile on the other buffer, so the key step is the longer of
-      // one tile's MMAs and one tile's softmax instead of their sum.
+      // wait P(j); O += P(j) V_j; free pair j + 1; S(j + 2) = Q K_{j+2}^T into
+      // the buffer P(j) came from (issue order: P V reads P(j) first) and
+      // commit it.  That commit also covers P V of tile j, so when no S(j + 2)
+      // is left it is issued all the same: it then only says "O holds P V up
+      // to tile j" (the last one: O final).  The softmax of tile j + 1 runs
+      // meanwhile on the other buffer, so the key step is the longer of one
+      // tile's MMAs and one tile's softmax instead of their sum.
       auto issue_qk1 = [&](int bf, uint32_t k_tile) {
 #pragma unroll
         for (int kk = 0; kk < D / 16; ++kk) {
@@ -389,12 +388,9 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
         if (lane0) {
           tc_fence_after();
           issue_pv1(j & 1, v_tile_of(u), j > 0);
-          umma_commit(bar_o_done);
           umma_commit(bar_empty + 8 * slot_of(u));
-          if (more2) {
-            issue_qk1(j & 1, k_tile_of(u + 1));
-            umma_commit(bar_s_full + 8 * (j & 1));
-          }
+          if (more2) issue_qk1(j & 1, k_tile_of(u + 1));
+          umma_commit(bar_s_full + 8 * (j & 1));   // S(j + 2), or only "P V of tile j done"
         }
         __syncwarp();
       }
@@ -477,9 +473,12 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
           m_used = tm;
         } else if (__any_sync(0xffffffffu, tm > m_used + 8.0f)) {
           // O must hold P V up to tile j-1, complete: with two tiles S(j) was
-          // announced after it; with one, wait for "O done" of tile j-1 (the
-          // barrier cannot be further ahead: P V of tile j needs this P).
-          if constexpr (kSingle) warp_wait(bar_o_done, (j - 1) & 1, abort, p.err, p.wait_limit);
+          // announced after it; with one, S(j+1) is (its commit follows P V
+          // of tile j-1; the barrier cannot be further ahead: S(j+3) needs
+          // this P).
+          if constexpr (kSingle)
+            warp_wait(bar_s_full + 8 * ((j + 1) & 1), static_cast<uint32_t>((j + 1) >> 1) & 1u, abort, p.err,
+                      p.wait_limit);
           const float m_new = fmaxf(m_used, tm);
           const float a = ex2_approx(m_used - m_new);
           m_used = m_new;
@@ -513,10 +512,10 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
       }
       bool ok;
       if constexpr (kSingle) {
-        // O final = "O done" of tile T-1; the barrier may be two phases behind
-        // (S(T-1) was issued before P V of tile T-2), so take them in order.
-        ok = (T < 2 || warp_wait(bar_o_done, (T - 2) & 1, abort, p.err, p.wait_limit)) &&
-             warp_wait(bar_o_done, (T - 1) & 1, abort, p.err, p.wait_limit);
+        // O final: the commit after P V of tile T-1 (buffer (T+1) & 1, the
+        // phase after S(T-1) on that buffer).
+        ok = warp_wait(bar_s_full + 8 * ((T + 1) & 1), static_cast<uint32_t>((T + 1) >> 1) & 1u, abort, p.err,
+                       p.wait_limit);
       } else {
         ok = warp_wait(bar_s, T & 1, abort, p.err, p.wait_limit);
       }
