@@ -264,7 +264,7 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
     }
     for (int i = 0; i < 2; ++i) {
       mbar_init(bar_s_full + 8 * i, 1);
-      mbar_init(bar_p_full + 8 * i, kBM);
+      mbar_init(bar_p_full + 8 * i, (!kSingle && i == 0) ? kBM + 1 : kBM);   // P_A: + the producer
     }
     *abort = 0;
     mbar_fence_init();
@@ -289,14 +289,36 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
   if (warp == kWarpProducer) {
     // ------------------------------------------------------------ producer
     // The whole warp runs the loop and waits (warp-uniform); lane 0 issues.
+    // Two-tile kernel: the MMA warp's wait for P_A(j) also covers "pair j+1
+    // has landed" (the barrier counts kBM + 1 arrivals): once that pair has
+    // landed and phase j-1 is over, so that this arrival cannot count towards
+    // it, the producer adds its arrival to phase j.  The MMA warp then waits
+    // once less per key tile.
+    auto landed = [&](int v) {                  // pair v landed -> phase v-1 of P_A
+      if (!warp_wait(bar_full + 8 * slot_of(v), static_cast<uint32_t>(use_of(v)) & 1u, abort, p.err,
+                     p.wait_limit))
+        return false;
+      if (v >= 2 && !warp_wait(bar_p_full, static_cast<uint32_t>(v - 2) & 1u, abort, p.err, p.wait_limit))
+        return false;
+      if (lane0) mbar_arrive(bar_p_full);
+      __syncwarp();
+      return true;
+    };
     int u = u_pre;
+    bool ok = true;
     for (; u <= T; ++u) {
+      if constexpr (!kSingle) {
+        if (!(ok = landed(u - 1))) break;       // u >= 2: pairs 0 .. u-1 are issued
+      }
       const int slot = slot_of(u), use = use_of(u);
       if (use > 0 && !warp_wait(bar_empty + 8 * slot, (use - 1) & 1, abort, p.err, p.wait_limit)) break;
       if (lane0) issue_pair(u);
       __syncwarp();
     }
     last_pair = u - 1;         // the loop breaks before issuing pair u
+    if constexpr (!kSingle) {
+      if (ok && u == T + 1) landed(T);          // the last pair (every earlier one arrived in the loop)
+    }
   } else if (warp == kWarpMma) {
     // ------------------------------------------------------------ MMA issuer
     // The whole warp runs the loop and waits (warp-uniform); lane 0 issues
@@ -412,8 +434,7 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
       int j = 0;
       for (; ok && j < T; ++j) {
         const bool more = j + 1 < T;
-        const int u = j + 1;                    // pair (V_j, K_{j+1})
-        if (!warp_wait(bar_full + 8 * (u & 1), phase_of(u), abort, p.err, p.wait_limit)) break;
+        const int u = j + 1;                    // pair (V_j, K_{j+1}), landed: P_A(j) says so
         for (int t = 0; t < n_tiles; ++t) {
           if (!warp_wait(bar_p_full + 8 * t, j & 1, abort, p.err, p.wait_limit)) { ok = false; break; }
           if (p.debug_skip_last_pv && !more) { ok = false; break; }   // the softmax's final wait must expire
