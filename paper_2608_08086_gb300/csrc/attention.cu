@@ -13,9 +13,10 @@
 //   warp 0     MMA issuer: the warp waits together, lane 0 issues.  Per K/V
 //              tile j: PV_A(j), QK_A(j+1), PV_B(j), QK_B(j+1), so the tensor
 //              pipe works on one tile while the other tile's softmax runs.  It
-//              waits on three barriers and commits three times per tile j:
-//              every wait or commit between two MMA batches idles the tensor
-//              pipe.  tcgen05.mma executes in issue order, so QK_X(j+1)
+//              waits on two barriers (P_A(j), which also says that the pair
+//              (V_j, K_{j+1}) has landed, and P_B(j)) and commits three times
+//              per tile j: every wait or commit between two MMA batches idles
+//              the tensor pipe.  tcgen05.mma executes in issue order, so QK_X(j+1)
 //              overwrites S_X only after PV_X(j) has read P_X(j), and the
 //              commit that announces S_X(j+1) also covers PV_X(j): when the
 //              softmax sees S_X(j+1), O_X is stable and may be rescaled without
@@ -23,7 +24,8 @@
 //   warp 1     TMA producer: Q_A, Q_B once, then pairs (V_{u-1}, K_u) of
 //              128-key tiles (u = 0 .. T; the first pair holds K_0 only, the
 //              last V_{T-1} only) through two pair slots, one full and one
-//              empty barrier per pair.
+//              empty barrier per pair.  It waits for each pair to land itself
+//              and adds one arrival to P_A of the key tile that reads it.
 //   warps 2-9  softmax: one warpgroup per tile.  Warp w reaches TMEM lanes
 //              32 (w % 4) .. 32 (w % 4) + 31, so lane i of warp w owns query
 //              row 32 (w % 4) + i and all 128 key columns of its tile, read
@@ -264,7 +266,7 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
     }
     for (int i = 0; i < 2; ++i) {
       mbar_init(bar_s_full + 8 * i, 1);
-      mbar_init(bar_p_full + 8 * i, (!kSingle && i == 0) ? kBM + 1 : kBM);   // P_A: + the producer
+      mbar_init(bar_p_full + 8 * i, (kSingle || i == 0) ? kBM + 1 : kBM);   // + the producer's arrival
     }
     *abort = 0;
     mbar_fence_init();
@@ -304,11 +306,30 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
       __syncwarp();
       return true;
     };
+    // One-tile kernel: the same for P(j) (buffer j % 2) and pair min(j+2, T),
+    // the pair the MMA warp reads next (K_{j+2}; for the last tiles V_{T-1}),
+    // once the buffer's previous phase (tile j-2) is over.
+    int next_j = 0;
+    auto landed1 = [&](int j) {
+      const int v = min(j + 2, T);
+      if (!warp_wait(bar_full + 8 * slot_of(v), static_cast<uint32_t>(use_of(v)) & 1u, abort, p.err,
+                     p.wait_limit))
+        return false;
+      if (j >= 2 &&
+          !warp_wait(bar_p_full + 8 * (j & 1), static_cast<uint32_t>((j - 2) >> 1) & 1u, abort, p.err, p.wait_limit))
+        return false;
+      if (lane0) mbar_arrive(bar_p_full + 8 * (j & 1));
+      __syncwarp();
+      return true;
+    };
     int u = u_pre;
     bool ok = true;
     for (; u <= T; ++u) {
       if constexpr (!kSingle) {
         if (!(ok = landed(u - 1))) break;       // u >= 2: pairs 0 .. u-1 are issued
+      } else {
+        while (ok && next_j < T && min(next_j + 2, T) <= u - 1) ok = landed1(next_j++);
+        if (!ok) break;
       }
       const int slot = slot_of(u), use = use_of(u);
       if (use > 0 && !warp_wait(bar_empty + 8 * slot, (use - 1) & 1, abort, p.err, p.wait_limit)) break;
@@ -316,8 +337,10 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
       __syncwarp();
     }
     last_pair = u - 1;         // the loop breaks before issuing pair u
-    if constexpr (!kSingle) {
-      if (ok && u == T + 1) landed(T);          // the last pair (every earlier one arrived in the loop)
+    if (ok && u == T + 1) {                     // every pair is issued: the arrivals left
+      if constexpr (!kSingle) landed(T);
+      else
+        while (ok && next_j < T) ok = landed1(next_j++);
     }
   } else if (warp == kWarpMma) {
     // ------------------------------------------------------------ MMA issuer
@@ -395,18 +418,12 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
       for (; ok && j < T; ++j) {
         const int u = j + 1;                  // pair (V_j, K_{j+1})
         const bool more2 = j + 2 < T;         // S(j + 2) to compute
-        // pair u was waited for S(j + 1), except the last pair (V_{T-1} only)
-        if (j + 1 == T && T > 1 && !warp_wait(bar_full + 8 * slot_of(u), phase_of(u), abort, p.err, p.wait_limit))
-          break;
+        // P(j) also says pair min(j + 2, T) has landed (the producer's arrival)
         if (!warp_wait(bar_p_full + 8 * (j & 1), static_cast<uint32_t>(j >> 1) & 1u, abort, p.err, p.wait_limit)) {
           ok = false;
           break;
         }
         if (p.debug_skip_last_pv && j + 1 == T) { ok = false; break; }   // the softmax's final wait must expire
-        if (more2 && !warp_wait(bar_full + 8 * slot_of(u + 1), phase_of(u + 1), abort, p.err, p.wait_limit)) {
-          ok = false;
-          break;
-        }
         if (lane0) {
           tc_fence_after();
           issue_pv1(j & 1, v_tile_of(u), j > 0);
