@@ -23,9 +23,11 @@
 //              a wait.
 //   warp 1     TMA producer: Q_A, Q_B once, then pairs (V_{u-1}, K_u) of
 //              128-key tiles (u = 0 .. T; the first pair holds K_0 only, the
-//              last V_{T-1} only) through two pair slots, one full and one
-//              empty barrier per pair.  It waits for each pair to land itself
-//              and adds one arrival to P_A of the key tile that reads it.
+//              last V_{T-1} only) through two pair slots, one full barrier
+//              per slot.  It waits for each pair to land itself and adds one
+//              arrival to P_A of the key tile that reads it, and it takes a
+//              slot as free from tile B's S barrier, whose commit after the
+//              key tile that last read the slot covers those reads.
 //   warps 2-9  softmax: one warpgroup per tile.  Warp w reaches TMEM lanes
 //              32 (w % 4) .. 32 (w % 4) + 31, so lane i of warp w owns query
 //              row 32 (w % 4) + i and all 128 key columns of its tile, read
@@ -108,8 +110,9 @@ struct Layout {
   static constexpr uint32_t kOffQ = 0;                      // Q_A, Q_B (Q only when kSingle)
   static constexpr uint32_t kOffKV = kOffQ + (kSingle ? 1 : 2) * kTile;
   static constexpr uint32_t kOffBar = kOffKV + kSlots * 2 * kTile;
-  // q_full, full[slots], empty[slots], s_full[2], p_full[2]
-  static constexpr int kBars = 1 + 2 * kSlots + 4;
+  // q_full, full[slots], s_full[2], p_full[2] (a pair slot is known free from
+  // the S barrier whose commit covers the pair's last reader)
+  static constexpr int kBars = 1 + kSlots + 4;
   static constexpr uint32_t kOffHolder = kOffBar + 8 * kBars;
   static constexpr uint32_t kOffAbort = kOffHolder + 4;
   static constexpr uint32_t kOffDrain = kOffAbort + 4;        // abort path: the MMA warp's MMAs done
@@ -228,8 +231,7 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
   const uint32_t bars = base + L::kOffBar;
   const uint32_t bar_q_full = bars;
   const uint32_t bar_full = bars + 8;                           // + 8 * slot
-  const uint32_t bar_empty = bar_full + 8 * L::kSlots;          // + 8 * slot
-  const uint32_t bar_s_full = bar_empty + 8 * L::kSlots;        // + 8 * tile (A = 0, B = 1)
+  const uint32_t bar_s_full = bar_full + 8 * L::kSlots;         // + 8 * tile (A = 0, B = 1)
   const uint32_t bar_p_full = bar_s_full + 16;                  // + 8 * tile: both halves of P written
   const uint32_t bar_drain = base + L::kOffDrain;
   uint32_t* holder = reinterpret_cast<uint32_t*>(gbase + L::kOffHolder);
@@ -262,7 +264,6 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
     mbar_init(bar_q_full, 1);
     for (int s = 0; s < L::kSlots; ++s) {
       mbar_init(bar_full + 8 * s, 1);
-      mbar_init(bar_empty + 8 * s, 1);
     }
     for (int i = 0; i < 2; ++i) {
       mbar_init(bar_s_full + 8 * i, 1);
@@ -325,14 +326,27 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
     int u = u_pre;
     bool ok = true;
     for (; u <= T; ++u) {
+      const int use = use_of(u);
       if constexpr (!kSingle) {
+        // Slot of pair u free: its previous pair u-2 was read by the MMAs of
+        // key step u-3 (or the prologue), which the last tile's S commit of
+        // that step covers (completion u-2).  Polled before the arrival that
+        // lets key step u-2 start, so that barrier cannot be two phases ahead.
+        if (!warp_wait(bar_s_full + 8 * (has_b ? 1 : 0), static_cast<uint32_t>(u - 2) & 1u, abort, p.err,
+                       p.wait_limit))
+          break;
         if (!(ok = landed(u - 1))) break;       // u >= 2: pairs 0 .. u-1 are issued
       } else {
         while (ok && next_j < T && min(next_j + 2, T) <= u - 1) ok = landed1(next_j++);
         if (!ok) break;
+        // Slot of pair u free: its previous pair u-3 was last read by P V of
+        // key step u-4 (or, for pair 0, by the prologue), which the commit
+        // announcing S(u-2) covers.  S(u) needs this very pair, so that
+        // buffer's barrier cannot be two phases ahead.
+        if (use > 0 && !warp_wait(bar_s_full + 8 * ((u - 2) & 1), static_cast<uint32_t>((u - 2) >> 1) & 1u, abort,
+                                  p.err, p.wait_limit))
+          break;
       }
-      const int slot = slot_of(u), use = use_of(u);
-      if (use > 0 && !warp_wait(bar_empty + 8 * slot, (use - 1) & 1, abort, p.err, p.wait_limit)) break;
       if (lane0) issue_pair(u);
       __syncwarp();
     }
@@ -401,7 +415,6 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
           tc_fence_after();
           issue_qk1(0, k_tile_of(0));
           umma_commit(bar_s_full);
-          umma_commit(bar_empty + 8 * slot_of(0));
         }
         __syncwarp();
         ok = warp_wait(bar_full + 8 * slot_of(1), phase_of(1), abort, p.err, p.wait_limit);
@@ -427,7 +440,6 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
         if (lane0) {
           tc_fence_after();
           issue_pv1(j & 1, v_tile_of(u), j > 0);
-          umma_commit(bar_empty + 8 * slot_of(u));
           if (more2) issue_qk1(j & 1, k_tile_of(u + 1));
           umma_commit(bar_s_full + 8 * (j & 1));   // S(j + 2), or only "P V of tile j done"
         }
@@ -444,7 +456,6 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
             issue_qk(t, k_tile_of(0));
             umma_commit(bar_s_full + 8 * t);
           }
-          umma_commit(bar_empty);               // pair 0 (K_0) read
         }
         __syncwarp();
       }
@@ -464,8 +475,6 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
           __syncwarp();
         }
         if (!ok) break;
-        if (lane0) umma_commit(bar_empty + 8 * (u & 1));
-        __syncwarp();
       }
       mma_done = ok && j == T;
     }
