@@ -10,7 +10,7 @@
 //
 // One CTA = two 128-row query tiles (A and B) of one (b, h) sharing every K/V
 // tile; 10 warps:
-//   warp 0     MMA issuer: the warp waits together, lane 0 issues.  Per K/V
+//   warp 0     MMA issuer: lane 0 waits and issues alone.  Per K/V
 //              tile j: PV_A(j), QK_A(j+1), PV_B(j), QK_B(j+1), so the tensor
 //              pipe works on one tile while the other tile's softmax runs.  It
 //              waits on two barriers (P_A(j), which also says that the pair
@@ -358,8 +358,10 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
     }
   } else if (warp == kWarpMma) {
     // ------------------------------------------------------------ MMA issuer
-    // The whole warp runs the loop and waits (warp-uniform); lane 0 issues
-    // every MMA and commit, so the warp never runs diverged for long.
+    // Lane 0 runs the schedule alone: its waits are single-thread bounded
+    // waits, and it issues every MMA and commit (measured a little faster
+    // than the whole warp waiting together and reconverging after each
+    // batch).
     constexpr uint32_t idesc_qk = idesc_bf16_f32(kBM, kBN, 0, 0);
     constexpr uint32_t idesc_pv = idesc_bf16_f32(kBM, D, 0, 1);
     const int n_tiles = has_b ? 2 : 1;
@@ -407,76 +409,73 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
           umma_ts(tmem + col_o(0), tmem + col_s(bf) + 64 * (kk >> 2) + (kk & 3) * 8,
                   sdesc_sw128(v_tile + kk * 2048, kChunkBytes, 1024), idesc_pv, (acc || kk > 0) ? 1u : 0u);
       };
-      // pairs 0 (K_0) and 1 (V_0, K_1): S(0) and S(1)
-      bool ok = warp_wait(bar_q_full, 0, abort, p.err, p.wait_limit) &&
-                warp_wait(bar_full, phase_of(0), abort, p.err, p.wait_limit);
-      if (ok) {
-        if (lane0) {
+      // pairs 0 (K_0) and 1 (V_0, K_1): S(0) and S(1).  Lane 0 alone runs
+      // the schedule (single-thread bounded waits); the other lanes wait for
+      // it at the end.
+      bool ok = true;
+      int j = 0;
+      if (lane0) {
+        ok = mbar_wait(bar_q_full, 0, abort, p.err, p.wait_limit) &&
+             mbar_wait(bar_full, phase_of(0), abort, p.err, p.wait_limit);
+        if (ok) {
           tc_fence_after();
           issue_qk1(0, k_tile_of(0));
           umma_commit(bar_s_full);
+          ok = mbar_wait(bar_full + 8 * slot_of(1), phase_of(1), abort, p.err, p.wait_limit);
         }
-        __syncwarp();
-        ok = warp_wait(bar_full + 8 * slot_of(1), phase_of(1), abort, p.err, p.wait_limit);
-      }
-      if (ok && T > 1) {
-        if (lane0) {
+        if (ok && T > 1) {
           tc_fence_after();
           issue_qk1(1, k_tile_of(1));
           umma_commit(bar_s_full + 8);
         }
-        __syncwarp();
-      }
-      int j = 0;
-      for (; ok && j < T; ++j) {
-        const int u = j + 1;                  // pair (V_j, K_{j+1})
-        const bool more2 = j + 2 < T;         // S(j + 2) to compute
-        // P(j) also says pair min(j + 2, T) has landed (the producer's arrival)
-        if (!warp_wait(bar_p_full + 8 * (j & 1), static_cast<uint32_t>(j >> 1) & 1u, abort, p.err, p.wait_limit)) {
-          ok = false;
-          break;
-        }
-        if (p.debug_skip_last_pv && j + 1 == T) { ok = false; break; }   // the softmax's final wait must expire
-        if (lane0) {
+        for (; ok && j < T; ++j) {
+          const int u = j + 1;                // pair (V_j, K_{j+1})
+          const bool more2 = j + 2 < T;       // S(j + 2) to compute
+          // P(j) also says pair min(j + 2, T) has landed (the producer's arrival)
+          if (!mbar_wait(bar_p_full + 8 * (j & 1), static_cast<uint32_t>(j >> 1) & 1u, abort, p.err, p.wait_limit)) {
+            ok = false;
+            break;
+          }
+          if (p.debug_skip_last_pv && j + 1 == T) { ok = false; break; }   // the softmax's final wait must expire
           tc_fence_after();
           issue_pv1(j & 1, v_tile_of(u), j > 0);
           if (more2) issue_qk1(j & 1, k_tile_of(u + 1));
           umma_commit(bar_s_full + 8 * (j & 1));   // S(j + 2), or only "P V of tile j done"
         }
-        __syncwarp();
       }
-      mma_done = ok && j == T;
+      __syncwarp();
+      mma_done = __shfl_sync(0xffffffffu, (ok && j == T) ? 1 : 0, 0) != 0;
     } else {
-      bool ok = warp_wait(bar_q_full, 0, abort, p.err, p.wait_limit) &&
-                warp_wait(bar_full, phase_of(0), abort, p.err, p.wait_limit);
-      if (ok) {
-        if (lane0) {
+      // Lane 0 alone runs the schedule (single-thread bounded waits); the
+      // other lanes wait for it at the end.
+      bool ok = true;
+      int j = 0;
+      if (lane0) {
+        ok = mbar_wait(bar_q_full, 0, abort, p.err, p.wait_limit) &&
+             mbar_wait(bar_full, phase_of(0), abort, p.err, p.wait_limit);
+        if (ok) {
           tc_fence_after();
           for (int t = 0; t < n_tiles; ++t) {
             issue_qk(t, k_tile_of(0));
             umma_commit(bar_s_full + 8 * t);
           }
         }
-        __syncwarp();
-      }
-      int j = 0;
-      for (; ok && j < T; ++j) {
-        const bool more = j + 1 < T;
-        const int u = j + 1;                    // pair (V_j, K_{j+1}), landed: P_A(j) says so
-        for (int t = 0; t < n_tiles; ++t) {
-          if (!warp_wait(bar_p_full + 8 * t, j & 1, abort, p.err, p.wait_limit)) { ok = false; break; }
-          if (p.debug_skip_last_pv && !more) { ok = false; break; }   // the softmax's final wait must expire
-          if (lane0) {
+        for (; ok && j < T; ++j) {
+          const bool more = j + 1 < T;
+          const int u = j + 1;                  // pair (V_j, K_{j+1}), landed: P_A(j) says so
+          for (int t = 0; t < n_tiles; ++t) {
+            if (!mbar_wait(bar_p_full + 8 * t, j & 1, abort, p.err, p.wait_limit)) { ok = false; break; }
+            if (p.debug_skip_last_pv && !more) { ok = false; break; }   // the softmax's final wait must expire
             tc_fence_after();
             issue_pv(t, v_tile_of(u), j > 0);
             if (more) issue_qk(t, k_tile_of(u));
-            umma_commit(bar_s_full + 8 * t);   // S_t(j+1) ready -- or, after the last tile, O_t final
+            umma_commit(bar_s_full + 8 * t);     // S_t(j+1) ready -- or, after the last tile, O_t final
           }
-          __syncwarp();
+          if (!ok) break;
         }
-        if (!ok) break;
       }
-      mma_done = ok && j == T;
+      __syncwarp();
+      mma_done = __shfl_sync(0xffffffffu, (ok && j == T) ? 1 : 0, 0) != 0;
     }
   } else {
     // ------------------------------------------------------------ softmax
