@@ -297,11 +297,15 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
     // landed and phase j-1 is over, so that this arrival cannot count towards
     // it, the producer adds its arrival to phase j.  The MMA warp then waits
     // once less per key tile.
-    auto landed = [&](int v) {                  // pair v landed -> phase v-1 of P_A
+    // In the loop, the slot poll just before (tile B's S commit of key step
+    // v-2) already implies that phase v-2 is over; only the last arrival,
+    // after the loop, waits for it explicitly.
+    auto landed = [&](int v, bool wait_prev) {  // pair v landed -> phase v-1 of P_A
       if (!warp_wait(bar_full + 8 * slot_of(v), static_cast<uint32_t>(use_of(v)) & 1u, abort, p.err,
                      p.wait_limit))
         return false;
-      if (v >= 2 && !warp_wait(bar_p_full, static_cast<uint32_t>(v - 2) & 1u, abort, p.err, p.wait_limit))
+      if (wait_prev && v >= 2 &&
+          !warp_wait(bar_p_full, static_cast<uint32_t>(v - 2) & 1u, abort, p.err, p.wait_limit))
         return false;
       if (lane0) mbar_arrive(bar_p_full);
       __syncwarp();
@@ -335,7 +339,7 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
         if (!warp_wait(bar_s_full + 8 * (has_b ? 1 : 0), static_cast<uint32_t>(u - 2) & 1u, abort, p.err,
                        p.wait_limit))
           break;
-        if (!(ok = landed(u - 1))) break;       // u >= 2: pairs 0 .. u-1 are issued
+        if (!(ok = landed(u - 1, false))) break;   // u >= 2: pairs 0 .. u-1 are issued
       } else {
         while (ok && next_j < T && min(next_j + 2, T) <= u - 1) ok = landed1(next_j++);
         if (!ok) break;
@@ -352,7 +356,7 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
     }
     last_pair = u - 1;         // the loop breaks before issuing pair u
     if (ok && u == T + 1) {                     // every pair is issued: the arrivals left
-      if constexpr (!kSingle) landed(T);
+      if constexpr (!kSingle) landed(T, true);
       else
         while (ok && next_j < T) ok = landed1(next_j++);
     }
