@@ -204,8 +204,11 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
   const int h = (unit / p.tiles_x) % p.Hq, b = unit / (p.tiles_x * p.Hq);
   const int tp = tpx / p.n_split, split = tpx % p.n_split;
   // Launched as a programmatic dependent of the stream's previous kernel: wait
-  // for it before reading anything it may have written (flags, Q/K/V).
-  asm volatile("griddepcontrol.wait;" ::: "memory");
+  // for it before reading anything it may have written (flags, Q/K/V).  With
+  // no flags to read, the wait is deferred to just before the first load (and
+  // taken by every thread after the set-up barrier), so the barrier set-up
+  // and TMEM allocation overlap the previous kernel's tail.
+  if (p.flags) asm volatile("griddepcontrol.wait;" ::: "memory");
   // Lets a programmatic dependent (the split merge, the next layer) be
   // scheduled once every CTA of this grid is resident; it still waits for
   // this grid's completion.
@@ -271,6 +274,7 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
     }
     *abort = 0;
     mbar_fence_init();
+    if (!p.flags) asm volatile("griddepcontrol.wait;" ::: "memory");
     tma_prefetch_map(&tmQ);
     mbar_arrive_expect_tx(bar_q_full, has_b ? 2 * L::kTile : L::kTile);
     for (int t = 0; t < (has_b ? 2 : 1); ++t)
@@ -285,6 +289,7 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
+  if (!p.flags) asm volatile("griddepcontrol.wait;" ::: "memory");
   const uint32_t tmem = *holder;
 
   int last_pair = -1;          // producer: the last pair whose loads were issued
