@@ -397,13 +397,15 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
     if constexpr (kSingle) {
       // One query tile, S double buffered: S(j) in buffer j & 1 (columns
       // col_s(j & 1), P(j) written over it), O in col_o(0).  Per key tile j:
-      // wait P(j); O += P(j) V_j; free pair j + 1; S(j + 2) = Q K_{j+2}^T into
-      // the buffer P(j) came from (issue order: P V reads P(j) first) and
-      // commit it.  That commit also covers P V of tile j, so when no S(j + 2)
-      // is left it is issued all the same: it then only says "O holds P V up
-      // to tile j" (the last one: O final).  The softmax of tile j + 1 runs
-      // meanwhile on the other buffer, so the key step is the longer of one
-      // tile's MMAs and one tile's softmax instead of their sum.
+      // wait P(j) (with the producer's arrival it also says that pair
+      // min(j + 2, T) has landed); O += P(j) V_j; S(j + 2) = Q K_{j+2}^T into
+      // the buffer P(j) came from (issue order: P V reads P(j) first); one
+      // commit.  That commit also covers P V of tile j, so it tells the
+      // producer that pair j + 1 is read and, when no S(j + 2) is left (it is
+      // issued all the same), says only "O holds P V up to tile j" (the last
+      // one: O final).  The softmax of tile j + 1 runs meanwhile on the other
+      // buffer, so the key step is the longer of one tile's MMAs and one
+      // tile's softmax instead of their sum.
       auto issue_qk1 = [&](int bf, uint32_t k_tile) {
 #pragma unroll
         for (int kk = 0; kk < D / 16; ++kk) {
