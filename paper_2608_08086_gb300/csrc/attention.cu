@@ -694,7 +694,7 @@ attn_combine_kernel(const float* __restrict__ ws_o, const float2* __restrict__ w
 // ------------------------------------------------------------------ host side
 
 constexpr int kMaxSplit = 16;
-constexpr int kMinSplitTiles = 8;   // fewer key tiles: no split
+constexpr int kMinSplitTiles = 16;  // fewer key tiles: no split
 
 int sm_count() {
   static int count[64] = {0};
@@ -709,22 +709,24 @@ struct SplitPlan {
   size_t bytes = 0;
 };
 
-// Splits the T key tiles when the grid (query tile pairs x heads x batch)
-// leaves SMs idle and the tiles are many enough to pay for the merge: as many
-// splits as whole grids fit on the SMs, none empty.  Measured on the GB300
-// (B 1, 32 heads, G 256): P 2048 (T 18) 38 -> 26 us, P 1024 (T 10) 26 -> 23 us,
-// while T <= 6 gains nothing over a CTA's fixed start-up and the merge.
-//
-// Before that, a grid of two-tile CTAs that would still fill at most half the
-// SMs runs one query tile per CTA instead: twice the CTAs, each key step
-// shorter (one tile's MMAs and softmax), for latency-bound launches.
+// First, one query tile per CTA (the one-tile kernel, S double buffered) when
+// a query range holds one tile anyway, or when two-tile CTAs would fill at
+// most half the SMs (twice the CTAs, for latency-bound launches).  Then, when
+// the grid still leaves SMs idle, the T key tiles are split across CTAs if
+// they are many enough to pay for the merge: as many splits as whole grids
+// fit on the SMs, none empty.  Measured on the GB300 with the one-tile kernel
+// (B 1, 32 heads, G 256, launches replayed from a CUDA graph): P 2048 (T 18)
+// 18.8 -> 17.4 us split in two, while P 1024 (T 10) is 12.3 us whole against
+// 14.2 us split and T 6 9.3 us against 12.3 us.
 SplitPlan split_plan(int B, int P, int G, int Hq, int D, int rows, int M) {
   SplitPlan sp;
   const int T = (P + kBN - 1) / kBN + (G + kBN - 1) / kBN;
   sp.per = T;
   const int sms = sm_count();
   const long long pairs = static_cast<long long>((rows + 2 * kBM - 1) / (2 * kBM)) * Hq * B;
-  if (sms > 0 && rows > kBM && 2 * pairs <= sms) sp.tiles_per_cta = 1;
+  // One tile per CTA (the one-tile kernel) when a query range has one tile
+  // anyway, or when two-tile CTAs would fill at most half the SMs.
+  if (sms > 0 && (rows <= kBM || 2 * pairs <= sms)) sp.tiles_per_cta = 1;
   const int rows_per_cta = sp.tiles_per_cta * kBM;
   const long long ctas = static_cast<long long>((rows + rows_per_cta - 1) / rows_per_cta) * Hq * B;
   if (ctas <= 0 || sms <= 0 || ctas >= sms || T < kMinSplitTiles) return sp;

@@ -63,9 +63,10 @@ ATTN_CASES = [
     (1, 300, 1, 4, 4, 64),         # G = 1
     (2, 256, 256, 2, 2, 128),      # several full tiles in both segments
     (1, 129, 130, 4, 1, 64),       # one-past-a-tile in both segments, GQA 4:1
-    (1, 640, 384, 7, 1, 128),      # GQA 7:1, 8 KV tiles (split over the key tiles)
-    (1, 1500, 70, 3, 1, 64),       # 13 KV tiles, ragged tails: 13 splits of one tile
-    (2, 1500, 70, 8, 2, 64),       # 13 KV tiles over 7 splits of 2 + 2 + ... + 1 tiles
+    (1, 640, 384, 7, 1, 128),      # GQA 7:1, 8 KV tiles, one-tile CTAs
+    (1, 1664, 384, 7, 1, 128),     # GQA 7:1, 16 KV tiles: split over the key tiles
+    (1, 1900, 70, 3, 1, 64),       # 16 KV tiles, ragged tails: 16 splits of one tile
+    (2, 2000, 70, 8, 2, 64),       # 17 KV tiles over 9 splits of 2 + 2 + ... + 1 tiles
 ]
 
 
@@ -88,8 +89,8 @@ def test_attn_step_matches_oracle(A, case, sharp, split):
     out = torch.empty(B, G, Hq, D, dtype=torch.bfloat16, device="cuda")
     lse = torch.empty(B, Hq, G, dtype=torch.float32, device="cuda")
     shape = A.make_shape(B, P, G, Hq, Hkv, D, scale)
-    if split and (P + 127) // 128 + (G + 127) // 128 >= 8:
-        # a grid that leaves SMs idle over 8+ key tiles: the tiles are split across CTAs and merged
+    if split and (P + 127) // 128 + (G + 127) // 128 >= 16:
+        # a grid that leaves SMs idle over 16+ key tiles: the tiles are split across CTAs and merged
         assert A.archer_attn_workspace_size(shape, G) > 0
     A.archer_attn_step(shape, q_resp, d["k_cache"], d["v_cache"], d["k_resp"], d["v_resp"], out, lse,
                        workspace=None if split else False)
