@@ -234,8 +234,10 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
   const uint32_t bars = base + L::kOffBar;
   const uint32_t bar_q_full = bars;
   const uint32_t bar_full = bars + 8;                           // + 8 * slot
-  const uint32_t bar_s_full = bar_full + 8 * L::kSlots;         // + 8 * tile (A = 0, B = 1)
-  const uint32_t bar_p_full = bar_s_full + 16;                  // + 8 * tile: both halves of P written
+  // S ready / P written, + 8 * tile (A = 0, B = 1); the one-tile kernel: + 8 * S buffer.
+  // P_A (and the one-tile kernel's P) also count the producer's "pair landed".
+  const uint32_t bar_s_full = bar_full + 8 * L::kSlots;
+  const uint32_t bar_p_full = bar_s_full + 16;
   const uint32_t bar_drain = base + L::kOffDrain;
   uint32_t* holder = reinterpret_cast<uint32_t*>(gbase + L::kOffHolder);
   volatile int* abort = reinterpret_cast<volatile int*>(gbase + L::kOffAbort);
