@@ -49,6 +49,11 @@
 // sum.  With one Q tile in shared memory there is room for three K/V pair
 // slots.  The S barrier's commit after each P V also tells the softmax when O
 // may be rescaled and, after the last one, that O is final.
+//
+// Two-tile launches with many CTAs' worth of work run attn_fwd_persist_kernel
+// instead: one CTA per SM walks the work items, so the set-up happens once
+// and the next item's Q tiles and first K/V pairs load while the current one
+// finishes (its comment gives the barrier phases across items).
 
 #include <cmath>
 #include <cstdio>
@@ -647,6 +652,371 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
   }
 }
 
+// Persistent two-tile kernel: one CTA per SM walks work items x = blockIdx.x,
+// blockIdx.x + gridDim.x, ... (a work item = two 128-query tiles of one
+// (b, h), exactly as one CTA of attn_fwd_kernel<D, false>), so that the CTA's
+// set-up happens once and the next item's Q tiles and first K/V pairs load
+// while the current item finishes.  Barrier phases run on across items: with
+// k the item's rank among this CTA's items and T key tiles per item, S_X and
+// the K/V pairs share one running index k (T + 1) + u (the item's S commits:
+// S(0) after the prologue, then one per key step; its pairs u = 0 .. T), and
+// P_X completes k T + j times.  Two more barriers per tile: "O final"
+// (committed after the item's last P V, with that step's S commit) and "O
+// drained" (the tile's softmax warpgroup, after its epilogue has read O); the
+// MMA warp waits for the latter before the next item's first P V.  Used for
+// two-tile launches without splits whose items all hold two tiles.
+template <int D>
+__global__ void __launch_bounds__(kThreads, 1)
+attn_fwd_persist_kernel(const __grid_constant__ CUtensorMap tmQ,
+                        const __grid_constant__ CUtensorMap tmKpR, const __grid_constant__ CUtensorMap tmVpR,
+                        const __grid_constant__ CUtensorMap tmKpC, const __grid_constant__ CUtensorMap tmVpC,
+                        const __grid_constant__ CUtensorMap tmKg, const __grid_constant__ CUtensorMap tmVg,
+                        const AttnParams p) {
+  using L = Layout<D, false>;
+  extern __shared__ uint8_t smem_raw[];
+  if (p.flags) asm volatile("griddepcontrol.wait;" ::: "memory");
+  asm volatile("griddepcontrol.launch_dependents;");
+
+  const int n_units = p.tiles_x * p.Hq * p.B;
+  const int n_p = (p.P + kBN - 1) / kBN;
+  const int n_g = (p.G + kBN - 1) / kBN;
+  const int T = n_p + n_g;                                       // key tiles per item (no splits)
+  // Item x -> (b, h, first query row); q0 >= M: nothing to do for it.
+  auto decode = [&](int x, int& b, int& h, bool& refresh) {
+    const int tp = x % p.tiles_x;
+    h = (x / p.tiles_x) % p.Hq;
+    b = x / (p.tiles_x * p.Hq);
+    refresh = p.flags ? (p.flags[b] != 0) : (p.default_refresh != 0);
+    return (refresh ? p.q_begin_refresh : p.q_begin_cached) + tp * 2 * kBM;
+  };
+
+  const uint32_t raw = smem_u32(smem_raw);
+  const uint32_t base = (raw + 1023u) & ~1023u;
+  uint8_t* gbase = smem_raw + (base - raw);
+  const uint32_t sQ = base + L::kOffQ;
+  const uint32_t sKV = base + L::kOffKV;
+  const uint32_t bars = base + L::kOffBar;
+  const uint32_t bar_q_full = bars;
+  const uint32_t bar_full = bars + 8;                            // + 8 * slot
+  const uint32_t bar_s_full = bar_full + 8 * L::kSlots;          // + 8 * tile
+  const uint32_t bar_p_full = bar_s_full + 16;                   // + 8 * tile; P_A also counts "pair landed"
+  const uint32_t bar_drain = base + L::kOffDrain;
+  const uint32_t bar_o_ready = bar_drain + 8;                    // + 8 * tile: O final for the item
+  const uint32_t bar_o_free = bar_o_ready + 16;                  // + 8 * tile: O read by the epilogue
+  const uint32_t bar_q_free = bar_o_free + 16;                   // the item's last Q K^T batch done
+  uint32_t* holder = reinterpret_cast<uint32_t*>(gbase + L::kOffHolder);
+  volatile int* abort = reinterpret_cast<volatile int*>(gbase + L::kOffAbort);
+
+  const int warp = threadIdx.x >> 5;
+  const bool lane0 = (threadIdx.x & 31) == 0;
+  auto slot_of = [](int g) { return g & 1; };
+  auto phase_of = [](int g) { return static_cast<uint32_t>(g >> 1) & 1u; };
+  if (warp == kWarpProducer && lane0) {
+    mbar_init(bar_q_full, 1);
+    for (int s = 0; s < L::kSlots; ++s) mbar_init(bar_full + 8 * s, 1);
+    for (int i = 0; i < 2; ++i) {
+      mbar_init(bar_s_full + 8 * i, 1);
+      mbar_init(bar_p_full + 8 * i, i == 0 ? kBM + 1 : kBM);
+      mbar_init(bar_o_ready + 8 * i, 1);
+      mbar_init(bar_o_free + 8 * i, kBM);
+    }
+    mbar_init(bar_q_free, 1);
+    *abort = 0;
+    mbar_fence_init();
+  }
+  if (warp == kWarpMma) {
+    tmem_alloc(smem_u32(holder), kTmemCols);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  if (!p.flags) asm volatile("griddepcontrol.wait;" ::: "memory");
+  const uint32_t tmem = *holder;
+  const int stride = static_cast<int>(gridDim.x);
+
+  int last_pair = -1;          // producer: the last pair (running index) whose loads were issued
+  int q_loads = 0;             // producer: Q loads issued
+  bool mma_done = false;
+  if (warp == kWarpProducer) {
+    // ------------------------------------------------------------ producer
+    // Pairs in running order g = k (T + 1) + u.  Before issuing pair g: its
+    // slot's previous pair g-2 was read by MMAs that S_B's completion g-2
+    // covers (for u = 1 that pair is the previous item's last, read by the
+    // P V whose "O final" commit covers it; S_B is not used there because the
+    // next item's prologue may already have moved it two phases on).  Then
+    // the item's Q tiles (u = 0; the same poll says the previous item's last
+    // Q K^T is done), then the arrival on P_A for pair g-1 (the key step that
+    // reads it may start; the poll just before says the phase before is
+    // over), then the loads.
+    bool ok = true;
+    int k = 0;
+    int g_prev_last = -1;      // running index of the previous issued pair
+    for (int x = blockIdx.x; ok && x < n_units; x += stride) {
+      int b, h;
+      bool refresh;
+      const int q0 = decode(x, b, h, refresh);
+      if (q0 >= p.M) continue;
+      const int kvh = h / (p.Hq / p.Hkv);
+      const CUtensorMap* mKp = refresh ? &tmKpR : &tmKpC;
+      const CUtensorMap* mVp = refresh ? &tmVpR : &tmVpC;
+      for (int u = 0; u <= T; ++u) {
+        const int g = k * (T + 1) + u;
+        if (u == 0) {
+          // the previous item's Q K^T batches are done: Q and pair g-2's slot are free
+          if (k >= 1 && !warp_wait(bar_q_free, static_cast<uint32_t>(k - 1) & 1u, abort, p.err, p.wait_limit)) {
+            ok = false;
+            break;
+          }
+        } else if (u == 1) {
+          if (k >= 1 && !warp_wait(bar_o_ready + 8, static_cast<uint32_t>(k - 1) & 1u, abort, p.err, p.wait_limit)) {
+            ok = false;
+            break;
+          }
+        } else {
+          if (!warp_wait(bar_s_full + 8, static_cast<uint32_t>(g - 2) & 1u, abort, p.err, p.wait_limit)) {
+            ok = false;
+            break;
+          }
+        }
+        if (u == 0) {
+          if (lane0) {
+            if (k == 0) tma_prefetch_map(&tmQ);
+            mbar_arrive_expect_tx(bar_q_full, 2 * L::kTile);
+            for (int t = 0; t < 2; ++t)
+              for (int c = 0; c < L::kChunks; ++c)
+                tma_load_4d(sQ + t * L::kTile + c * kChunkBytes, &tmQ, bar_q_full, c * 64, h, q0 + t * kBM, b);
+          }
+          __syncwarp();
+          ++q_loads;
+        }
+        // pair g-1 landed -> its key step's P_A phase (pairs u = 0 hold K_0
+        // only and are waited by the MMA warp itself; an item's last pair
+        // arrived right after it was issued)
+        if (u >= 2) {
+          if (!warp_wait(bar_full + 8 * slot_of(g_prev_last), phase_of(g_prev_last), abort, p.err, p.wait_limit)) {
+            ok = false;
+            break;
+          }
+          if (lane0) mbar_arrive(bar_p_full);
+          __syncwarp();
+        }
+        if (lane0) {
+          const int slot = slot_of(g);
+          const bool has_v = u >= 1, has_k = u < T;
+          mbar_arrive_expect_tx(bar_full + 8 * slot, (has_v && has_k ? 2 : 1) * L::kTile);
+          for (int part = has_v ? 0 : 1; part < (has_k ? 2 : 1); ++part) {
+            const int j = part == 0 ? u - 1 : u;                // key tile
+            const bool in_prompt = j < n_p;
+            const int row = in_prompt ? j * kBN : (j - n_p) * kBN;
+            const CUtensorMap* map = in_prompt ? (part == 0 ? mVp : mKp) : (part == 0 ? &tmVg : &tmKg);
+            const uint32_t dst = sKV + (2 * slot + part) * L::kTile;
+            for (int c = 0; c < L::kChunks; ++c)
+              tma_load_4d(dst + c * kChunkBytes, map, bar_full + 8 * slot, c * 64, kvh, row, b);
+          }
+        }
+        __syncwarp();
+        last_pair = g;
+        g_prev_last = g;
+      }
+      // the item's last pair: its arrival at once, after the phase before it
+      // (no slot poll orders it; the next item's first poll is on "Q free")
+      if (ok && !*abort) {
+        const int pa = k * T + T - 1;                           // its P_A phase
+        ok = warp_wait(bar_full + 8 * slot_of(g_prev_last), phase_of(g_prev_last), abort, p.err, p.wait_limit) &&
+             (pa == 0 || warp_wait(bar_p_full, static_cast<uint32_t>(pa - 1) & 1u, abort, p.err, p.wait_limit));
+        if (ok && lane0) mbar_arrive(bar_p_full);
+        __syncwarp();
+      }
+      ++k;
+    }
+  } else if (warp == kWarpMma) {
+    // ------------------------------------------------------------ MMA issuer
+    // Lane 0 alone.  Per item: wait for Q and pair k (T + 1) (K_0), S(0) of
+    // both tiles; per key step j: wait P_X (k T + j; P_A also says the pair
+    // landed), before the item's first P V also "O drained" of the previous
+    // item, then P_X V_j and Q_X K_{j+1}^T, commit S_X; after the last step
+    // also "O final".
+    constexpr uint32_t idesc_qk = idesc_bf16_f32(kBM, kBN, 0, 0);
+    constexpr uint32_t idesc_pv = idesc_bf16_f32(kBM, D, 0, 1);
+    auto issue_qk = [&](int t, uint32_t k_tile) {
+      const uint32_t q_tile = sQ + t * L::kTile;
+#pragma unroll
+      for (int kk = 0; kk < D / 16; ++kk) {
+        const uint32_t off = (kk >> 2) * kChunkBytes + (kk & 3) * 32;
+        umma_ss(tmem + col_s(t), sdesc_sw128(q_tile + off, 16, 1024), sdesc_sw128(k_tile + off, 16, 1024),
+                idesc_qk, kk > 0 ? 1u : 0u);
+      }
+    };
+    auto issue_pv = [&](int t, uint32_t v_tile, bool acc) {
+#pragma unroll
+      for (int kk = 0; kk < 8; ++kk)
+        umma_ts(tmem + col_o(t), tmem + col_s(t) + 64 * (kk >> 2) + (kk & 3) * 8,
+                sdesc_sw128(v_tile + kk * 2048, kChunkBytes, 1024), idesc_pv, (acc || kk > 0) ? 1u : 0u);
+    };
+    auto v_tile_of = [&](int g) { return sKV + 2 * slot_of(g) * L::kTile; };
+    auto k_tile_of = [&](int g) { return sKV + (2 * slot_of(g) + 1) * L::kTile; };
+    bool ok = true;
+    if (lane0) {
+      int k = 0;
+      for (int x = blockIdx.x; ok && x < n_units; x += stride) {
+        int b, h;
+        bool refresh;
+        if (decode(x, b, h, refresh) >= p.M) continue;
+        const int g0 = k * (T + 1);
+        ok = mbar_wait(bar_q_full, static_cast<uint32_t>(k) & 1u, abort, p.err, p.wait_limit) &&
+             mbar_wait(bar_full + 8 * slot_of(g0), phase_of(g0), abort, p.err, p.wait_limit);
+        if (!ok) break;
+        tc_fence_after();
+        for (int t = 0; t < 2; ++t) {
+          issue_qk(t, k_tile_of(g0));
+          umma_commit(bar_s_full + 8 * t);
+        }
+        if (T == 1) umma_commit(bar_q_free);
+        for (int j = 0; ok && j < T; ++j) {
+          const bool more = j + 1 < T;
+          const int g = g0 + j + 1;                             // pair (V_j, K_{j+1})
+          for (int t = 0; t < 2; ++t) {
+            if (p.debug_skip_last_pv && !more) { ok = false; break; }   // the softmax's wait for O must expire
+            if (!mbar_wait(bar_p_full + 8 * t, static_cast<uint32_t>(k * T + j) & 1u, abort, p.err,
+                           p.wait_limit) ||
+                (j == 0 && k >= 1 &&
+                 !mbar_wait(bar_o_free + 8 * t, static_cast<uint32_t>(k - 1) & 1u, abort, p.err, p.wait_limit))) {
+              ok = false;
+              break;
+            }
+            tc_fence_after();
+            issue_pv(t, v_tile_of(g), j > 0);
+            if (more) issue_qk(t, k_tile_of(g));
+            umma_commit(bar_s_full + 8 * t);
+            if (!more) umma_commit(bar_o_ready + 8 * t);
+            if (t == 1 && j + 2 == T) umma_commit(bar_q_free);     // the item's last Q K^T batch
+          }
+        }
+        ++k;
+      }
+    }
+    __syncwarp();
+    mma_done = __shfl_sync(0xffffffffu, ok ? 1 : 0, 0) != 0;
+  } else {
+    // ------------------------------------------------------------ softmax
+    // As in attn_fwd_kernel<D, false>, per item: S_X(j) is S_X's completion
+    // k (T + 1) + j; O final is "O final" k; after the epilogue the warpgroup
+    // arrives on "O drained".
+    const int t = (warp - kWarpSoftmax0) >> 2;
+    const int r = (warp & 3) * 32 + (threadIdx.x & 31);
+    const uint32_t t_lane = tmem + (static_cast<uint32_t>((warp & 3) * 32) << 16);
+    const uint32_t colS = col_s(t), colO = col_o(t);
+    const uint32_t bar_s = bar_s_full + 8 * t;
+    const uint32_t bar_ph = bar_p_full + 8 * t;
+    const float sl2 = p.scale_log2;
+    auto rescale_o = [&](float a) {
+#pragma unroll 1
+      for (int c0 = 0; c0 < D; c0 += 16) {
+        uint32_t o[16];
+        tmem_ld_16(t_lane + colO + c0, o);
+#pragma unroll
+        for (int kq = 0; kq < 16; ++kq) o[kq] = __float_as_uint(__uint_as_float(o[kq]) * a);
+        tmem_st_16(t_lane + colO + c0, o);
+      }
+    };
+    int k = 0;
+    for (int x = blockIdx.x; x < n_units && !*abort; x += stride) {
+      int b, h;
+      bool refresh;
+      const int q0 = decode(x, b, h, refresh);
+      if (q0 >= p.M) continue;
+      float m_used = -INFINITY;
+      float2 l2 = make_float2(0.f, 0.f);
+      for (int j = 0; j < T; ++j) {
+        warp_wait(bar_s, static_cast<uint32_t>(k * (T + 1) + j) & 1u, abort, p.err, p.wait_limit);
+        tc_fence_after();
+        const int valid = j < n_p ? min(kBN, p.P - j * kBN) : min(kBN, p.G - (j - n_p) * kBN);
+        float xs[128];
+        load_scores128(t_lane + colS, valid, xs);
+        const float tm = max128(xs) * sl2;
+        if (j == 0) {
+          m_used = tm;
+        } else if (__any_sync(0xffffffffu, tm > m_used + 8.0f)) {
+          // O holds P V up to tile j-1, complete (S(j) was announced after it).
+          const float m_new = fmaxf(m_used, tm);
+          const float a = ex2_approx(m_used - m_new);
+          m_used = m_new;
+          l2.x *= a;
+          l2.y *= a;
+          rescale_o(a);
+        }
+        const float2 neg_m = make_float2(-m_used, -m_used);
+        const float2 slv = make_float2(sl2, sl2);
+        float2 acc[2] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+          uint32_t pk[16];
+#pragma unroll
+          for (int kq = 0; kq < 16; ++kq) {
+            const float2 y = ffma2(make_float2(xs[32 * q + 2 * kq], xs[32 * q + 2 * kq + 1]), slv, neg_m);
+            const float2 pr = make_float2(ex2_approx(y.x), ex2_approx(y.y));
+            acc[kq & 1] = fadd2(acc[kq & 1], pr);
+            pk[kq] = pack_bf16x2(pr.x, pr.y);
+          }
+          tmem_st_16_async(t_lane + colS + 64 * (q >> 1) + 16 * (q & 1), pk);
+        }
+        tmem_wait_st();
+        l2 = fadd2(l2, fadd2(acc[0], acc[1]));
+        tc_fence_before();
+        mbar_arrive(bar_ph);
+      }
+      const bool ok = warp_wait(bar_o_ready + 8 * t, static_cast<uint32_t>(k) & 1u, abort, p.err, p.wait_limit);
+      tc_fence_after();
+      const float l_sum = l2.x + l2.y;
+      const int q = q0 + t * kBM + r;
+      const bool live = ok && q < p.M;
+      const float inv_l = 1.0f / l_sum;
+      __nv_bfloat16* orow = p.out + ((static_cast<size_t>(b) * p.M + q) * p.Hq + h) * D;
+#pragma unroll
+      for (int c0 = 0; c0 < D; c0 += 32) {
+        uint32_t o[32];
+        tmem_ld_32(t_lane + colO + c0, o);
+        uint32_t w[16];
+#pragma unroll
+        for (int kq = 0; kq < 16; ++kq)
+          w[kq] = pack_bf16x2(__uint_as_float(o[2 * kq]) * inv_l, __uint_as_float(o[2 * kq + 1]) * inv_l);
+        if (live) {
+          uint4* dst = reinterpret_cast<uint4*>(orow + c0);
+#pragma unroll
+          for (int v = 0; v < 4; ++v) dst[v] = make_uint4(w[4 * v], w[4 * v + 1], w[4 * v + 2], w[4 * v + 3]);
+        }
+      }
+      if (live && p.lse)
+        p.lse[(static_cast<size_t>(b) * p.Hq + h) * p.M + q] = (m_used + log2f(l_sum)) * 0.69314718055994531f;
+      tc_fence_before();
+      mbar_arrive(bar_o_free + 8 * t);
+      ++k;
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  const bool aborted = *abort != 0;
+  if (warp == kWarpMma) {
+    if (aborted || !mma_done) {
+      if (lane0) {
+        mbar_init(bar_drain, 1);
+        mbar_fence_init();
+        umma_commit(bar_drain);
+      }
+      __syncwarp();
+      drain_wait(bar_drain, 0, p.wait_limit);
+    }
+    __syncwarp();
+    tc_fence_after();
+    tmem_dealloc(tmem, kTmemCols);
+  } else if (warp == kWarpProducer && aborted) {
+    if (q_loads > 0) drain_wait(bar_q_full, static_cast<uint32_t>(q_loads - 1) & 1u, p.wait_limit);
+    for (int g = max(0, last_pair - 1); g <= last_pair; ++g) drain_wait(bar_full + 8 * slot_of(g), phase_of(g), p.wait_limit);
+  }
+}
+
 // Merges the key-range splits of one output row (b, q, h): with m_s the
 // split's running max (log2 units), l_s its row sum and O_s its unnormalised
 // output, out = sum_s 2^(m_s - m) O_s / sum_s 2^(m_s - m) l_s, m = max_s m_s.
@@ -780,6 +1150,9 @@ int launch_d(const AttnCall& c, cudaStream_t stream) {
     if (e == cudaSuccess)
       e = cudaFuncSetAttribute(attn_fwd_kernel<D, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                (int)Layout<D, true>::kSmemBytes);
+    if (e == cudaSuccess)
+      e = cudaFuncSetAttribute(attn_fwd_persist_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                               (int)Layout<D, false>::kSmemBytes + 40);
     if (e != cudaSuccess) return cuda_status(e, "cudaFuncSetAttribute(attention)");
     configured_device = dev;
   }
@@ -846,7 +1219,22 @@ int launch_d(const AttnCall& c, cudaStream_t stream) {
     if (r > 0 && 2 * r <= sms) tail = r;
   }
   prm.n_unit_ctas = static_cast<int>(units) - tail;
-  const dim3 grid(static_cast<unsigned>(units + tail));
+  // The persistent two-tile kernel (one CTA per SM walking the items) when no
+  // item is split or single: the query ranges in use are whole tile pairs,
+  // and either no last wave would run as single tiles or every SM has four
+  // items or more.
+  bool persist = false;
+  if (sp.tiles_per_cta == 2 && sp.n_split == 1 && sms > 0 && units > sms) {
+    const bool uses_c = c.flags || !c.default_refresh, uses_r = c.flags || c.default_refresh;
+    const bool whole = (!uses_c || (c.M - c.q_begin_cached) % (2 * kBM) == 0) &&
+                       (!uses_r || (c.M - c.q_begin_refresh) % (2 * kBM) == 0);
+    persist = whole && (tail == 0 || units >= 4LL * sms);
+  }
+  if (persist) {
+    tail = 0;
+    prm.n_unit_ctas = static_cast<int>(units);
+  }
+  const dim3 grid(static_cast<unsigned>(persist ? sms : units + tail));
   // A programmatic dependent launch: its launch latency overlaps the previous
   // kernel on the stream, which every CTA waits for before its first read.
   // One query tile per CTA runs the one-tile kernel (S double buffered).
@@ -854,16 +1242,19 @@ int launch_d(const AttnCall& c, cudaStream_t stream) {
   cudaLaunchConfig_t lc = {};
   lc.gridDim = grid;
   lc.blockDim = dim3(kThreads);
-  lc.dynamicSmemBytes = single ? Layout<D, true>::kSmemBytes : Layout<D, false>::kSmemBytes;
+  lc.dynamicSmemBytes = single ? Layout<D, true>::kSmemBytes
+                               : (persist ? Layout<D, false>::kSmemBytes + 40 : Layout<D, false>::kSmemBytes);
   lc.stream = stream;
   cudaLaunchAttribute la[1];
   la[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
   la[0].val.programmaticStreamSerializationAllowed = 1;
   lc.attrs = la;
   lc.numAttrs = 1;
-  int st = cuda_status(single ? cudaLaunchKernelEx(&lc, attn_fwd_kernel<D, true>, mq, mkr, mvr, mkc, mvc, mkg, mvg, prm)
-                              : cudaLaunchKernelEx(&lc, attn_fwd_kernel<D, false>, mq, mkr, mvr, mkc, mvc, mkg, mvg, prm),
-                       "attention launch");
+  int st = cuda_status(
+      single    ? cudaLaunchKernelEx(&lc, attn_fwd_kernel<D, true>, mq, mkr, mvr, mkc, mvc, mkg, mvg, prm)
+      : persist ? cudaLaunchKernelEx(&lc, attn_fwd_persist_kernel<D>, mq, mkr, mvr, mkc, mvc, mkg, mvg, prm)
+                : cudaLaunchKernelEx(&lc, attn_fwd_kernel<D, false>, mq, mkr, mvr, mkc, mvc, mkg, mvg, prm),
+      "attention launch");
   if (st || sp.n_split == 1) return st;
   // The merge is a programmatic dependent launch: it is scheduled while the
   // attention grid still runs and waits for it on the device.
