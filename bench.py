@@ -57,7 +57,7 @@ MEASURED_TRAFFIC = {
     # (kernel, workload): DRAM bytes read + written per launch from one ncu capture
     # (dram__bytes_read.sum + dram__bytes_write.sum), valid only while the kernel's
     # sources hash to sha16 (sha256 over the listed files, first 16 hex digits).
-    ("attn_step", "gqa_long"): {"bytes": 248524032, "sha16": "d42b1488ae18a66f",
+    ("attn_step", "gqa_long"): {"bytes": 244445952, "sha16": "e38e70afa9da843d",
                                 "sources": ["attention.cu", "archer_device.cuh", "tmem_ldst.cuh"]},
     ("scores", "gqa_long"): {"bytes": 2496017920, "sha16": "f609be40559ef555",
                              "sources": ["decode_scores.cu", "archer_device.cuh"]},
@@ -745,7 +745,7 @@ def main():
             "speedup_vs_refresh_every_step": value / eager_value,
             "eager_steps_per_s": eager_value,
             "attention": att,
-            "roofline": {"bound": "tensor", "kernel": "attn_fwd_kernel<128, false>", "launches": "cached step",
+            "roofline": {"bound": "tensor", "kernel": "attn_fwd_persist_kernel<128>", "launches": "cached step",
                          "flops_per_launch": flops_step_launch, "achieved": achieved, "peak": peak_tf,
                          "unit": "TFLOP/s", "frac": achieved / peak_tf,
                          "traffic": measured_traffic("attn_step", wl.name),
