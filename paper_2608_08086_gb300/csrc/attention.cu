@@ -55,6 +55,7 @@
 // and the next item's Q tiles and first K/V pairs load while the current one
 // finishes (its comment gives the barrier phases across items).
 
+#include <atomic>
 #include <cmath>
 #include <cstdio>
 #include <cstdlib>
@@ -1068,12 +1069,16 @@ attn_combine_kernel(const float* __restrict__ ws_o, const float2* __restrict__ w
 constexpr int kMaxSplit = 16;
 constexpr int kMinSplitTiles = 16;  // fewer key tiles: no split
 
+// The current device's SM count, queried once per device (host threads may
+// race on the first query; they store the same value).
 int sm_count() {
-  static int count[64] = {0};
+  static std::atomic<int> count[64];
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return 0;
-  if (count[dev] == 0) cudaDeviceGetAttribute(&count[dev], cudaDevAttrMultiProcessorCount, dev);
-  return count[dev];
+  int c = count[dev].load(std::memory_order_relaxed);
+  if (c == 0 && cudaDeviceGetAttribute(&c, cudaDevAttrMultiProcessorCount, dev) == cudaSuccess)
+    count[dev].store(c, std::memory_order_relaxed);
+  return c;
 }
 
 struct SplitPlan {
@@ -1141,10 +1146,16 @@ bool make_map(CUtensorMap* map, const void* ptr, int B, int L, int H, int D) {
 
 template <int D>
 int launch_d(const AttnCall& c, cudaStream_t stream) {
-  static int configured_device = -1;
+  // Shared-memory limits are per device; setting them twice (two host threads
+  // on a first call) is harmless.
+  static std::atomic<bool> configured[64];
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess) return cuda_status(cudaGetLastError(), "cudaGetDevice");
-  if (configured_device != dev) {
+  if (dev < 0 || dev >= 64) {
+    set_error("device ordinal %d out of range", dev);
+    return ARCHER_ERR_UNSUPPORTED;
+  }
+  if (!configured[dev].load(std::memory_order_acquire)) {
     cudaError_t e = cudaFuncSetAttribute(attn_fwd_kernel<D, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                          (int)Layout<D, false>::kSmemBytes);
     if (e == cudaSuccess)
@@ -1154,7 +1165,7 @@ int launch_d(const AttnCall& c, cudaStream_t stream) {
       e = cudaFuncSetAttribute(attn_fwd_persist_kernel<D>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                (int)Layout<D, false>::kSmemBytes + 40);
     if (e != cudaSuccess) return cuda_status(e, "cudaFuncSetAttribute(attention)");
-    configured_device = dev;
+    configured[dev].store(true, std::memory_order_release);
   }
   CUtensorMap mq, mkr, mvr, mkc, mvc, mkg, mvg;
   bool ok = make_map(&mq, c.q, c.B, c.M, c.Hq, D) && make_map(&mkg, c.kg, c.B, c.G, c.Hkv, D) &&
