@@ -38,6 +38,12 @@ def test_threshold_is_inclusive_for_accept():
     g = np.array([[M, M]], np.int32)
     g2, _ = O.decoder_update(g, np.array([0.9, 0.1]), np.array([4, 5]), np.zeros(2), 0.9, 0.05, M)
     np.testing.assert_array_equal(g2, [[4, M]])
+    # two positions exactly at the threshold: both accepted (the progress rule
+    # alone would take one)
+    g2, ch = O.decoder_update(np.array([[M, M, M]], np.int32), np.array([0.9, 0.9, 0.3]), np.array([4, 5, 6]),
+                              np.zeros(3), 0.9, 0.05, M)
+    np.testing.assert_array_equal(g2, [[4, 5, M]])
+    np.testing.assert_array_equal(ch, [[1, 1, 0]])
 
 
 def test_closed_loop_trajectory_makes_progress_and_rolls_back():

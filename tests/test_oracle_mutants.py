@@ -1,13 +1,20 @@
 """The oracle's pins catch the slips they are meant to catch.
 
-Each case below plants one plausible mistake in a copy of the oracle's C++
-source (a dropped key segment, a flipped sign, a wrong GQA index, a
-transposed operand, the scale applied twice, a wrong tie-break, an
-off-by-one in the refresh rule, ...), builds that copy into a temporary
-library, and runs every pin of tests/test_oracle_pins.py and the oracle
-fixtures of tests/test_golden.py against it: at least one must fail.  The
-unmodified oracle passes the same pins in those files, so a mutant that
+Each case below plants one plausible mistake in a copy of the oracle's
+source and runs the oracle's pins against the mutant: at least one must
+fail.  The unmodified oracle passes the same pins, so a mutant that
 survived would mean the pins leave that part of the oracle unchecked.
+
+* C++ kernels of the oracle (a dropped key segment, a flipped sign, a wrong
+  GQA index, a transposed operand, the scale applied twice, a wrong
+  tie-break, an off-by-one in the refresh rule, ...): the mutated copy is
+  built into a temporary library and run against every pin of
+  tests/test_oracle_pins.py and the oracle fixtures of tests/test_golden.py.
+* Python parts (the rollback decoder, the Algorithm 1 driver, the
+  staleness bound): the mutated module source is executed into a fresh
+  module, the one mutated function is patched into the oracle's module, and
+  tests/test_decoder_oracle.py, tests/test_trajectory_oracle.py and
+  tests/test_staleness_oracle.py run against it.
 
 Every planted change keeps every memory access in bounds (the transposed
 reads index an [D, N] view of the same N x D buffer), so a mutant can only
@@ -15,13 +22,19 @@ compute a wrong value, never crash the test process.  CPU only.
 """
 import inspect
 import os
+import types
 
 import pytest
 
 from oracle import oracle as O
+from oracle import staleness as OS
+from oracle import trajectory as OT
 
+import test_decoder_oracle
 import test_golden
 import test_oracle_pins
+import test_staleness_oracle
+import test_trajectory_oracle
 
 # (name, original text, planted text): the original must occur exactly once.
 MUTANTS = [
@@ -53,11 +66,41 @@ MUTANTS = [
 ]
 
 
-def _pins():
+# (module, function, name, original text, planted text) for the Python parts.
+PY_MUTANTS = [
+    (O, "decoder_update", "accept_strict", "if mp[b, i] >= tau_accept:", "if mp[b, i] > tau_accept:"),
+    (O, "decoder_update", "remask_wrong_direction", "elif cp[b, i] < tau_remask:", "elif cp[b, i] > tau_remask:"),
+    (O, "decoder_update", "remask_inclusive", "elif cp[b, i] < tau_remask:", "elif cp[b, i] <= tau_remask:"),
+    (O, "decoder_update", "progress_highest_index_on_ties", "if mp[b, i] > best:", "if mp[b, i] >= best:"),
+    (O, "decoder_update", "progress_rule_dropped", "if not accepted and best_i >= 0:", "if False:"),
+    (OT, "run", "cached_step_reads_fresh_prompt",
+     'O.attn_step(x["q_all"][:, P:], x["k_cache"], x["v_cache"],',
+     'O.attn_step(x["q_all"][:, P:], x["k_new"], x["v_new"],'),
+    (OT, "run", "anchor_not_carried", "dist, flag, g_anchor, age = O.should_refresh(",
+     "dist, flag, _anchor, age = O.should_refresh("),
+    (OT, "run", "redrawn_query_rows_offset", 'x["q_all"][bidx, P + pos] = _f64(rows["q"])',
+     'x["q_all"][bidx, pos] = _f64(rows["q"])'),
+    (OT, "run", "response_k_not_redrawn", 'x["k_resp"][bidx, pos] = _f64(rows["k"])',
+     'x["k_resp"][bidx, pos] = x["k_resp"][bidx, pos]'),
+    (OT, "run", "refresh_ignores_flags", "scale, flags=flag,", "scale, flags=None,"),
+    (OS, "gamma", "gamma_drops_value_term", "return b_e * alpha_row * (av + scale * qn * ak * vmax)",
+     "return b_e * alpha_row * (scale * qn * ak * vmax)"),
+    (OS, "gamma", "gamma_drops_key_term", "return b_e * alpha_row * (av + scale * qn * ak * vmax)",
+     "return b_e * alpha_row * av"),
+    (OS, "curve", "curve_compares_cached_with_itself", "o_fresh, _ = O.attn_step(q, kf, vf, kg, vg, scale)",
+     "o_fresh, _ = O.attn_step(q, kc, vc, kg, vg, scale)"),
+    (OS, "curve", "bound_linear_in_distance", "gam * math.sqrt(d)", "gam * d"),
+]
+
+PIN_MODULES = (test_oracle_pins, test_golden)
+PY_PIN_MODULES = (test_decoder_oracle, test_trajectory_oracle, test_staleness_oracle)
+
+
+def _pins(modules=PIN_MODULES):
     """Every oracle pin as (label, zero-argument callable), parametrized cases
     expanded; tests that need fixtures (the GPU ones) are left out."""
     out = []
-    for mod in (test_oracle_pins, test_golden):
+    for mod in modules:
         for name, fn in sorted(vars(mod).items()):
             if not name.startswith("test_") or not callable(fn):
                 continue
@@ -78,13 +121,15 @@ def _pins():
     return out
 
 
-def _caught_by(pins):
+def _caught_by(pins, first=False):
     failed = []
     for label, call in pins:
         try:
             call()
         except AssertionError:
             failed.append(label)
+            if first:
+                break
     return failed
 
 
@@ -92,6 +137,8 @@ def test_pin_battery_is_complete():
     labels = [label for label, _ in _pins()]
     assert sum(label.startswith("test_oracle_pins.") for label in labels) >= 25
     assert sum(label.startswith("test_golden.") for label in labels) >= 3
+    py = [label for label, _ in _pins(PY_PIN_MODULES)]
+    assert len(py) >= 16
 
 
 @pytest.mark.parametrize("name,orig,planted", MUTANTS, ids=[m[0] for m in MUTANTS])
@@ -105,5 +152,24 @@ def test_planted_slip_fails_a_pin(name, orig, planted, tmp_path, monkeypatch):
     monkeypatch.setattr(O, "_SRC", path)
     monkeypatch.setattr(O, "_BUILD", os.path.join(tmp_path, "_build"))
     monkeypatch.setattr(O, "_lib", None)
-    caught = _caught_by(_pins())
+    caught = _caught_by(_pins(), first=True)
     assert caught, f"no oracle pin fails when the oracle has the slip '{name}'"
+
+
+def _mutated_function(mod, fn_name, orig, planted):
+    """fn_name from a fresh copy of mod whose source has orig replaced."""
+    with open(mod.__file__) as f:
+        src = f.read()
+    fn_src = inspect.getsource(getattr(mod, fn_name))
+    assert src.count(orig) == 1 and fn_src.count(orig) == 1, "mutation site is not unique in its function"
+    fresh = types.ModuleType(mod.__name__ + "_mutant")
+    fresh.__file__ = mod.__file__
+    exec(compile(src.replace(orig, planted), mod.__file__, "exec"), fresh.__dict__)
+    return getattr(fresh, fn_name)
+
+
+@pytest.mark.parametrize("mod,fn_name,name,orig,planted", PY_MUTANTS, ids=[m[2] for m in PY_MUTANTS])
+def test_planted_slip_in_python_oracle_fails_a_pin(mod, fn_name, name, orig, planted, monkeypatch):
+    monkeypatch.setattr(mod, fn_name, _mutated_function(mod, fn_name, orig, planted))
+    caught = _caught_by(_pins(PY_PIN_MODULES), first=True)
+    assert caught, f"no oracle pin fails when {mod.__name__}.{fn_name} has the slip '{name}'"

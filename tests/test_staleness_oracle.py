@@ -53,3 +53,27 @@ def test_error_scales_like_sqrt_d():
     errs = np.mean([[e for _, e, _ in S.curve(SHAPE, ds, seed=s)] for s in range(6)], axis=0)
     r = errs / np.sqrt(ds)
     assert r.max() < 1.5 * r.min()
+
+
+def test_gamma_closed_form():
+    # pieces whose norms are known by hand: embedding diameter 2 ([1, 0] to
+    # [-1, 0]), largest alpha row norm 5 ([3, 4]), ||A_K||_2 = 2, ||A_V||_2 = 3
+    # (diagonal), max ||q_i||_2 = 2, max |v| = 4 (response V), s = 1/4:
+    # Gamma = 2 * 5 * (3 + 0.25 * 2 * 2 * 4) = 70
+    model = {"emb": np.array([[1.0, 0.0], [0.0, 1.0], [-1.0, 0.0]]),
+             "alpha": np.array([[3.0, 4.0], [0.0, 1.0]]),
+             "a_k": np.diag([2.0, 1.0]), "a_v": np.diag([0.5, 3.0])}
+    q = np.array([[[0.6, 0.8]], [[0.0, 2.0]]])
+    v_cache = np.array([[1.5, -1.0]])
+    v_resp = np.array([[-4.0, 0.5]])
+    assert S.gamma(model, q, v_cache, v_resp, 0.25) == pytest.approx(70.0, rel=1e-14)
+
+
+def test_reported_bound_grows_like_sqrt_d():
+    # the bound the curve reports is Gamma sqrt(D_t) (Eq. theory-radius-bound):
+    # zero at D = 0, and its ratios between distances are those of sqrt(D)
+    ds = [0, 1, 4, 9, 25]
+    pts = S.curve(SHAPE, ds, seed=5)
+    assert pts[0][2] == 0.0
+    for d, _, bound in pts[1:]:
+        assert bound / pts[1][2] == pytest.approx(math.sqrt(d), rel=1e-12)
