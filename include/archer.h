@@ -98,6 +98,43 @@ int archer_prompt_refresh(const archer_shape* shape, const void* q_all, const vo
                           const uint8_t* refresh_flags, void* workspace, size_t ws_bytes,
                           void* stream);
 
+/* Launch plan of one attention call, for tests and capacity planning.
+ * op: ARCHER_PLAN_ATTN_STEP (archer_attn_step), ARCHER_PLAN_REFRESH_ALL
+ * (archer_prompt_refresh with refresh_flags NULL) or ARCHER_PLAN_REFRESH_FLAGS
+ * (with flags).  ws_bytes: the 16-byte aligned workspace the call would get
+ * (0: none).  sm_count: SMs of the GPU to plan for; <= 0 queries the current
+ * device.  With sm_count > 0 the call is host arithmetic only (no CUDA call,
+ * no GPU needed).  The attention calls launch exactly this plan: 128-row
+ * query tiles, one or two per work item; the key range of an item split when
+ * the grid leaves SMs idle and the workspace suffices (a merge kernel then
+ * follows); a persistent grid of sm_count CTAs when items of two whole tiles
+ * outnumber the SMs.  Writes *plan (zeros for batch 0); returns ARCHER_OK, or
+ * ARCHER_ERR_ARG / ARCHER_ERR_UNSUPPORTED for a shape the calls would reject.
+ * Sec. 4.1 defines the attention this plans; the plan itself is this
+ * library's. */
+enum {
+  ARCHER_PLAN_ATTN_STEP = 0,
+  ARCHER_PLAN_REFRESH_ALL = 1,
+  ARCHER_PLAN_REFRESH_FLAGS = 2
+};
+enum {
+  ARCHER_KERNEL_TWO_TILE = 0,    /* one CTA per item of two query tiles */
+  ARCHER_KERNEL_ONE_TILE = 1,    /* one CTA per query tile (S double buffered) */
+  ARCHER_KERNEL_PERSISTENT = 2   /* one CTA per SM walking two-tile items */
+};
+typedef struct archer_attn_plan {
+  int kernel;                /* ARCHER_KERNEL_*                                   */
+  int tiles_per_cta;         /* query tiles per work item: 1 or 2                 */
+  int n_split;               /* key-range splits per item (> 1: merge kernel)     */
+  int key_tiles_per_split;   /* 128-key tiles one split walks                     */
+  int work_items;            /* items over (sequence, head, query range, split)   */
+  int grid;                  /* CTAs of the attention launch                      */
+  int single_tail;           /* trailing one-tile CTAs of a two-tile launch       */
+  size_t split_workspace;    /* workspace bytes a split wants (0: no split wanted) */
+} archer_attn_plan;
+int archer_attn_plan_query(const archer_shape* shape, int op, size_t ws_bytes, int sm_count,
+                           archer_attn_plan* plan);
+
 /* Scratch bytes that let archer_attn_step / archer_prompt_refresh split the
  * key tiles of a launch over n_queries (= G or N) query rows per sequence:
  * n_split * B * Hq * n_queries * (4 D + 8), n_split chosen from the SM count;

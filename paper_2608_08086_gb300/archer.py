@@ -58,6 +58,16 @@ class archer_step_desc(ctypes.Structure):
                 ("attn_workspace_bytes", ctypes.c_size_t)]
 
 
+class archer_attn_plan(ctypes.Structure):
+    _fields_ = [("kernel", ctypes.c_int), ("tiles_per_cta", ctypes.c_int), ("n_split", ctypes.c_int),
+                ("key_tiles_per_split", ctypes.c_int), ("work_items", ctypes.c_int), ("grid", ctypes.c_int),
+                ("single_tail", ctypes.c_int), ("split_workspace", ctypes.c_size_t)]
+
+
+ARCHER_PLAN_ATTN_STEP, ARCHER_PLAN_REFRESH_ALL, ARCHER_PLAN_REFRESH_FLAGS = 0, 1, 2
+ARCHER_KERNEL_TWO_TILE, ARCHER_KERNEL_ONE_TILE, ARCHER_KERNEL_PERSISTENT = 0, 1, 2
+
+
 def _load():
     if not os.path.exists(LIB_PATH):
         raise ImportError(f"{LIB_PATH} is missing: build it with paper_2608_08086_gb300.build.build() "
@@ -67,6 +77,7 @@ def _load():
     sp = ctypes.POINTER(archer_shape)
     L.archer_attn_step.argtypes = [sp, vp, vp, vp, vp, vp, vp, vp, vp, sz, vp]
     L.archer_prompt_refresh.argtypes = [sp, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, vp, sz, vp]
+    L.archer_attn_plan_query.argtypes = [sp, i, sz, i, ctypes.POINTER(archer_attn_plan)]
     L.archer_attn_workspace_size.argtypes = [sp, i]
     L.archer_attn_workspace_size.restype = sz
     L.archer_decode_scores.argtypes = [i, i, i, i, vp, ctypes.c_int64, vp, vp, vp, vp, vp, vp, vp, sz, vp]
@@ -88,7 +99,7 @@ def _load():
     L.archer_step_graph_destroy.argtypes = [vp]
     for name in ("archer_attn_step", "archer_prompt_refresh", "archer_decode_scores", "archer_should_refresh",
                  "archer_cache_rewrite", "archer_check_device", "archer_version", "archer_step_graph_create",
-                 "archer_decoder_update", "archer_scatter_rows",
+                 "archer_decoder_update", "archer_scatter_rows", "archer_attn_plan_query",
                  "archer_step_graph_launch", "archer_step_graph_destroy"):
         getattr(L, name).restype = ctypes.c_int
     return L
@@ -207,6 +218,16 @@ def archer_prompt_refresh(shape: archer_shape, q_all, k_prompt_new, v_prompt_new
         _ptr(out, bf, "out"), _ptr(lse, torch.float32, "lse"), _ptr(k_cache, bf, "k_cache"),
         _ptr(v_cache, bf, "v_cache"), _ptr(refresh_flags, torch.uint8, "refresh_flags"), _ptr(ws, None, "workspace"),
         ctypes.c_size_t(0 if ws is None else ws.numel() * ws.element_size()), _stream(stream)))
+
+
+def archer_attn_plan_query(shape: archer_shape, op: int = ARCHER_PLAN_ATTN_STEP, ws_bytes: int = 0,
+                           sm_count: int = 0) -> dict:
+    """The launch an attention call makes (kernel, split, grid); with
+    sm_count > 0 host arithmetic only, no GPU needed."""
+    plan = archer_attn_plan()
+    _raise(lib.archer_attn_plan_query(ctypes.byref(shape), int(op), ctypes.c_size_t(int(ws_bytes)), int(sm_count),
+                                      ctypes.byref(plan)))
+    return {name: int(getattr(plan, name)) for name, _ in archer_attn_plan._fields_}
 
 
 def archer_attn_workspace_size(shape: archer_shape, n_queries: int) -> int:

@@ -87,6 +87,32 @@ int check_ptrs(const char* names, std::initializer_list<const void*> ptrs) {
   return ARCHER_OK;
 }
 
+static_assert(ARCHER_KERNEL_TWO_TILE == kPlanTwoTile && ARCHER_KERNEL_ONE_TILE == kPlanOneTile &&
+                  ARCHER_KERNEL_PERSISTENT == kPlanPersistent,
+              "public kernel ids follow the planner's");
+
+// The fields of an archer_attn_step call that do not depend on its buffers.
+AttnCall step_call(const archer_shape* s, float scale) {
+  AttnCall c{};
+  c.B = s->batch; c.P = s->prompt_len; c.G = s->resp_len;
+  c.Hq = s->n_heads; c.Hkv = s->n_kv_heads; c.D = s->head_dim;
+  c.scale = scale;
+  c.M = c.G;
+  c.flags = nullptr; c.default_refresh = 0;
+  c.q_begin_refresh = 0; c.q_begin_cached = 0;
+  return c;
+}
+
+// The same for archer_prompt_refresh: every position is a query of a
+// refreshed sequence, rows P.. of a sequence whose flag is clear.
+AttnCall refresh_call(const archer_shape* s, float scale, const uint8_t* flags) {
+  AttnCall c = step_call(s, scale);
+  c.M = c.P + c.G;
+  c.flags = flags; c.default_refresh = 1;
+  c.q_begin_refresh = 0; c.q_begin_cached = c.P;
+  return c;
+}
+
 }  // namespace
 }  // namespace archer
 
@@ -103,17 +129,12 @@ int archer_attn_step(const archer_shape* shape, const void* q_resp, const void* 
   if ((st = check_ptrs("q_resp, k_resp, v_resp, out", {q_resp, k_resp, v_resp, out}))) return st;
   if (shape->prompt_len > 0 && (st = check_ptrs("k_cache, v_cache", {k_cache, v_cache}))) return st;
   if (lse && (reinterpret_cast<uintptr_t>(lse) & 3u)) { set_error("lse is not 4-byte aligned"); return ARCHER_ERR_ARG; }
-  AttnCall c{};
-  c.B = shape->batch; c.P = shape->prompt_len; c.G = shape->resp_len;
-  c.Hq = shape->n_heads; c.Hkv = shape->n_kv_heads; c.D = shape->head_dim;
-  c.scale = scale;
-  c.q = q_resp; c.M = c.G;
+  AttnCall c = step_call(shape, scale);
+  c.q = q_resp;
   c.kp_refresh = k_cache; c.vp_refresh = v_cache;
   c.kp_cached = k_cache; c.vp_cached = v_cache;
   c.kg = k_resp; c.vg = v_resp;
   c.out = out; c.lse = lse;
-  c.flags = nullptr; c.default_refresh = 0;
-  c.q_begin_refresh = 0; c.q_begin_cached = 0;
   c.ws = workspace; c.ws_bytes = ws_bytes;
   return attn_launch(c, static_cast<cudaStream_t>(stream));
 }
@@ -131,17 +152,12 @@ int archer_prompt_refresh(const archer_shape* shape, const void* q_all, const vo
     return st;
   if (lse && (reinterpret_cast<uintptr_t>(lse) & 3u)) { set_error("lse is not 4-byte aligned"); return ARCHER_ERR_ARG; }
   const cudaStream_t s = static_cast<cudaStream_t>(stream);
-  AttnCall c{};
-  c.B = shape->batch; c.P = shape->prompt_len; c.G = shape->resp_len;
-  c.Hq = shape->n_heads; c.Hkv = shape->n_kv_heads; c.D = shape->head_dim;
-  c.scale = scale;
-  c.q = q_all; c.M = c.P + c.G;
+  AttnCall c = refresh_call(shape, scale, refresh_flags);
+  c.q = q_all;
   c.kp_refresh = k_prompt_new; c.vp_refresh = v_prompt_new;
   c.kp_cached = k_cache; c.vp_cached = v_cache;
   c.kg = k_resp; c.vg = v_resp;
   c.out = out; c.lse = lse;
-  c.flags = refresh_flags; c.default_refresh = 1;
-  c.q_begin_refresh = 0; c.q_begin_cached = c.P;
   c.ws = workspace; c.ws_bytes = ws_bytes;
   if ((st = attn_launch(c, s))) return st;
   if (c.P == 0) return ARCHER_OK;
@@ -150,6 +166,33 @@ int archer_prompt_refresh(const archer_shape* shape, const void* q_all, const vo
   if (!copy_k && !copy_v) return ARCHER_OK;
   return cache_rewrite_launch(c.B, per_seq, copy_k ? k_prompt_new : nullptr, copy_v ? v_prompt_new : nullptr,
                               copy_k ? k_cache : nullptr, copy_v ? v_cache : nullptr, refresh_flags, s);
+}
+
+int archer_attn_plan_query(const archer_shape* shape, int op, size_t ws_bytes, int sm_count,
+                           archer_attn_plan* plan) {
+  if (!plan) { set_error("plan is NULL"); return ARCHER_ERR_ARG; }
+  *plan = archer_attn_plan{};
+  float scale = 0.f;
+  int st = check_shape(shape, &scale);
+  if (st) return st;
+  static const uint8_t some_flags = 1;     // never read: only "flags given" matters
+  AttnCall c;
+  if (op == ARCHER_PLAN_ATTN_STEP) c = step_call(shape, scale);
+  else if (op == ARCHER_PLAN_REFRESH_ALL) c = refresh_call(shape, scale, nullptr);
+  else if (op == ARCHER_PLAN_REFRESH_FLAGS) c = refresh_call(shape, scale, &some_flags);
+  else { set_error("unknown plan op %d", op); return ARCHER_ERR_ARG; }
+  if (c.B == 0) return ARCHER_OK;                 // the calls launch nothing
+  AttnPlan pl;
+  if ((st = attn_plan(c, ws_bytes, sm_count, &pl))) return st;
+  plan->kernel = pl.kernel;
+  plan->tiles_per_cta = pl.tiles_per_cta;
+  plan->n_split = pl.n_split;
+  plan->key_tiles_per_split = pl.per;
+  plan->work_items = pl.units;
+  plan->grid = pl.grid;
+  plan->single_tail = pl.tail;
+  plan->split_workspace = pl.split_bytes;
+  return ARCHER_OK;
 }
 
 size_t archer_attn_workspace_size(const archer_shape* shape, int n_queries) {

@@ -47,6 +47,25 @@ int attn_launch(const AttnCall& c, cudaStream_t stream);
 // CTAs (0 when the launch would not split: its grid already fills the GPU).
 size_t attn_workspace_bytes(int B, int P, int G, int Hq, int D, int M);
 
+// The launch an attention call makes on a GPU of `sms` SMs (<= 0: the
+// current device's count) with `usable_ws` bytes of aligned workspace.  Host
+// arithmetic only when sms > 0 (no CUDA call); the launch reads its kernel,
+// grid and split from it.
+constexpr int kPlanTwoTile = 0, kPlanOneTile = 1, kPlanPersistent = 2;
+struct AttnPlan {
+  int kernel = kPlanTwoTile;
+  int tiles_per_cta = 2;     // 128-row query tiles per work item
+  int n_split = 1;           // key-range splits per item (> 1: a merge kernel follows)
+  int per = 0;               // key tiles per split
+  int tiles_x = 0;           // items per (sequence, head), splits included
+  int units = 0;             // items over the launch
+  int tail = 0;              // trailing one-tile CTAs of a two-tile launch
+  int n_unit_ctas = 0;       // CTAs that run whole items
+  int grid = 0;              // CTAs launched
+  size_t split_bytes = 0;    // workspace the split wants (0: no split wanted)
+};
+int attn_plan(const AttnCall& c, size_t usable_ws, int sms, AttnPlan* plan);
+
 int cache_rewrite_launch(int B, size_t bytes_per_seq, const void* k_src, const void* v_src,
                          void* k_dst, void* v_dst, const uint8_t* flags, cudaStream_t stream);
 

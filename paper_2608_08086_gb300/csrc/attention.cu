@@ -1095,11 +1095,10 @@ struct SplitPlan {
 // (B 1, 32 heads, G 256, launches replayed from a CUDA graph): P 2048 (T 18)
 // 18.8 -> 17.4 us split in two, while P 1024 (T 10) is 12.3 us whole against
 // 14.2 us split and T 6 9.3 us against 12.3 us.
-SplitPlan split_plan(int B, int P, int G, int Hq, int D, int rows, int M) {
+SplitPlan split_plan(int B, int P, int G, int Hq, int D, int rows, int M, int sms) {
   SplitPlan sp;
   const int T = (P + kBN - 1) / kBN + (G + kBN - 1) / kBN;
   sp.per = T;
-  const int sms = sm_count();
   const long long pairs = static_cast<long long>((rows + 2 * kBM - 1) / (2 * kBM)) * Hq * B;
   // One tile per CTA (the one-tile kernel) when a query range has one tile
   // anyway, or when two-tile CTAs would fill at most half the SMs.
@@ -1196,61 +1195,28 @@ int launch_d(const AttnCall& c, cudaStream_t stream) {
   prm.out = static_cast<__nv_bfloat16*>(c.out);
   prm.lse = c.lse;
   prm.err = device_error_word();
-  // Query tiles needed by the longest query range (a refreshed sequence's).
-  const int rows = c.M - (c.flags || c.default_refresh ? c.q_begin_refresh : c.q_begin_cached);
-  SplitPlan sp = split_plan(c.B, c.P, c.G, c.Hq, D, rows, c.M);
-  prm.tiles_per_cta = sp.tiles_per_cta;
-  if (sp.n_split > 1 && (!c.ws || c.ws_bytes < sp.bytes || (reinterpret_cast<uintptr_t>(c.ws) & 15u))) {
-    sp.n_split = 1;                                 // no (usable) workspace: one CTA per tile pair
-    sp.per = (c.P + kBN - 1) / kBN + (c.G + kBN - 1) / kBN;
-  }
-  prm.n_split = sp.n_split;
-  prm.tiles_per_split = sp.per;
+  const size_t usable_ws = (c.ws && !(reinterpret_cast<uintptr_t>(c.ws) & 15u)) ? c.ws_bytes : 0;
+  AttnPlan pl;
+  int st = attn_plan(c, usable_ws, 0, &pl);
+  if (st) return st;
+  prm.tiles_per_cta = pl.tiles_per_cta;
+  prm.n_split = pl.n_split;
+  prm.tiles_per_split = pl.per;
   prm.ws_o = nullptr;
   prm.ws_ml = nullptr;
-  if (sp.n_split > 1) {
+  if (pl.n_split > 1) {
     prm.ws_o = static_cast<float*>(c.ws);
     prm.ws_ml = reinterpret_cast<float2*>(static_cast<char*>(c.ws) +
-                                          static_cast<size_t>(sp.n_split) * c.B * c.Hq * c.M * D * 4);
+                                          static_cast<size_t>(pl.n_split) * c.B * c.Hq * c.M * D * 4);
   }
-  const int rows_per_cta = sp.tiles_per_cta * kBM;
   prm.B = c.B;
-  prm.tiles_x = ((rows + rows_per_cta - 1) / rows_per_cta) * sp.n_split;
-  const long long units = static_cast<long long>(prm.tiles_x) * c.Hq * c.B;
-  if (units > 0x3FFFFFFFll) {
-    set_error("too many attention work units (%lld)", units);
-    return ARCHER_ERR_UNSUPPORTED;
-  }
-  // A last wave of tile pairs at most half full runs as one wave of single
-  // tiles instead: each of its SMs then finishes in about 0.7 of a pair's time.
-  int tail = 0;
-  const int sms = sm_count();
-  if (sp.n_split == 1 && sp.tiles_per_cta == 2 && sms > 0 && units > sms) {
-    const int r = static_cast<int>(units % sms);
-    if (r > 0 && 2 * r <= sms) tail = r;
-  }
-  prm.n_unit_ctas = static_cast<int>(units) - tail;
-  // The persistent two-tile kernel (one CTA per SM walking the items) when no
-  // item is split or single: the query ranges in use are whole tile pairs,
-  // and either no last wave would run as single tiles or every SM has three
-  // items or more (measured: the 32-layer trajectory's 512 items, 3.4 per SM,
-  // 93.3 -> 91.1 us against flat pairs with single-tile tails).
-  bool persist = false;
-  if (sp.tiles_per_cta == 2 && sp.n_split == 1 && sms > 0 && units > sms) {
-    const bool uses_c = c.flags || !c.default_refresh, uses_r = c.flags || c.default_refresh;
-    const bool whole = (!uses_c || (c.M - c.q_begin_cached) % (2 * kBM) == 0) &&
-                       (!uses_r || (c.M - c.q_begin_refresh) % (2 * kBM) == 0);
-    persist = whole && (tail == 0 || units >= 3LL * sms);
-  }
-  if (persist) {
-    tail = 0;
-    prm.n_unit_ctas = static_cast<int>(units);
-  }
-  const dim3 grid(static_cast<unsigned>(persist ? sms : units + tail));
+  prm.tiles_x = pl.tiles_x;
+  prm.n_unit_ctas = pl.n_unit_ctas;
+  const bool single = pl.kernel == kPlanOneTile, persist = pl.kernel == kPlanPersistent;
+  const dim3 grid(static_cast<unsigned>(pl.grid));
   // A programmatic dependent launch: its launch latency overlaps the previous
   // kernel on the stream, which every CTA waits for before its first read.
   // One query tile per CTA runs the one-tile kernel (S double buffered).
-  const bool single = sp.tiles_per_cta == 1;
   cudaLaunchConfig_t lc = {};
   lc.gridDim = grid;
   lc.blockDim = dim3(kThreads);
@@ -1262,12 +1228,12 @@ int launch_d(const AttnCall& c, cudaStream_t stream) {
   la[0].val.programmaticStreamSerializationAllowed = 1;
   lc.attrs = la;
   lc.numAttrs = 1;
-  int st = cuda_status(
+  st = cuda_status(
       single    ? cudaLaunchKernelEx(&lc, attn_fwd_kernel<D, true>, mq, mkr, mvr, mkc, mvc, mkg, mvg, prm)
       : persist ? cudaLaunchKernelEx(&lc, attn_fwd_persist_kernel<D>, mq, mkr, mvr, mkc, mvc, mkg, mvg, prm)
                 : cudaLaunchKernelEx(&lc, attn_fwd_kernel<D, false>, mq, mkr, mvr, mkc, mvc, mkg, mvg, prm),
       "attention launch");
-  if (st || sp.n_split == 1) return st;
+  if (st || pl.n_split == 1) return st;
   // The merge is a programmatic dependent launch: it is scheduled while the
   // attention grid still runs and waits for it on the device.
   const long long threads = static_cast<long long>(c.B) * c.M * c.Hq * (D / 8);
@@ -1281,7 +1247,7 @@ int launch_d(const AttnCall& c, cudaStream_t stream) {
   cfg.attrs = attr;
   cfg.numAttrs = 1;
   return cuda_status(cudaLaunchKernelEx(&cfg, attn_combine_kernel<D>, static_cast<const float*>(prm.ws_o),
-                                        static_cast<const float2*>(prm.ws_ml), sp.n_split, c.B, c.Hq, c.M, c.flags,
+                                        static_cast<const float2*>(prm.ws_ml), pl.n_split, c.B, c.Hq, c.M, c.flags,
                                         c.default_refresh, c.q_begin_refresh, c.q_begin_cached, prm.out, prm.lse),
                      "attention combine launch");
 }
@@ -1304,7 +1270,56 @@ __global__ void cache_rewrite_kernel(const uint4* __restrict__ k_src, const uint
 }  // namespace
 
 size_t attn_workspace_bytes(int B, int P, int G, int Hq, int D, int M) {
-  return split_plan(B, P, G, Hq, D, M, M).bytes;
+  return split_plan(B, P, G, Hq, D, M, M, sm_count()).bytes;
+}
+
+int attn_plan(const AttnCall& c, size_t usable_ws, int sms, AttnPlan* pl) {
+  *pl = AttnPlan{};
+  if (sms <= 0) sms = sm_count();
+  // Query tiles needed by the longest query range (a refreshed sequence's).
+  const int rows = c.M - (c.flags || c.default_refresh ? c.q_begin_refresh : c.q_begin_cached);
+  SplitPlan sp = split_plan(c.B, c.P, c.G, c.Hq, c.D, rows, c.M, sms);
+  pl->split_bytes = sp.bytes;
+  if (sp.n_split > 1 && usable_ws < sp.bytes) {
+    sp.n_split = 1;                                 // no (usable) workspace: one CTA per tile pair
+    sp.per = (c.P + kBN - 1) / kBN + (c.G + kBN - 1) / kBN;
+  }
+  pl->tiles_per_cta = sp.tiles_per_cta;
+  pl->n_split = sp.n_split;
+  pl->per = sp.per;
+  const int rows_per_cta = sp.tiles_per_cta * kBM;
+  pl->tiles_x = ((rows + rows_per_cta - 1) / rows_per_cta) * sp.n_split;
+  const long long units = static_cast<long long>(pl->tiles_x) * c.Hq * c.B;
+  if (units > 0x3FFFFFFFll) {
+    set_error("too many attention work units (%lld)", units);
+    return ARCHER_ERR_UNSUPPORTED;
+  }
+  pl->units = static_cast<int>(units);
+  // A last wave of tile pairs at most half full runs as one wave of single
+  // tiles instead: each of its SMs then finishes in about 0.7 of a pair's time.
+  int tail = 0;
+  if (sp.n_split == 1 && sp.tiles_per_cta == 2 && sms > 0 && units > sms) {
+    const int r = static_cast<int>(units % sms);
+    if (r > 0 && 2 * r <= sms) tail = r;
+  }
+  // The persistent two-tile kernel (one CTA per SM walking the items) when no
+  // item is split or single: the query ranges in use are whole tile pairs,
+  // and either no last wave would run as single tiles or every SM has three
+  // items or more (measured: the 32-layer trajectory's 512 items, 3.4 per SM,
+  // 93.3 -> 91.1 us against flat pairs with single-tile tails).
+  bool persist = false;
+  if (sp.tiles_per_cta == 2 && sp.n_split == 1 && sms > 0 && units > sms) {
+    const bool uses_c = c.flags || !c.default_refresh, uses_r = c.flags || c.default_refresh;
+    const bool whole = (!uses_c || (c.M - c.q_begin_cached) % (2 * kBM) == 0) &&
+                       (!uses_r || (c.M - c.q_begin_refresh) % (2 * kBM) == 0);
+    persist = whole && (tail == 0 || units >= 3LL * sms);
+  }
+  if (persist) tail = 0;
+  pl->tail = tail;
+  pl->n_unit_ctas = static_cast<int>(units) - tail;
+  pl->kernel = sp.tiles_per_cta == 1 ? kPlanOneTile : (persist ? kPlanPersistent : kPlanTwoTile);
+  pl->grid = persist ? sms : static_cast<int>(units) + tail;
+  return ARCHER_OK;
 }
 
 int attn_launch(const AttnCall& c, cudaStream_t stream) {
