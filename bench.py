@@ -525,6 +525,26 @@ def run_e2e(wl, steps, warmup, dist_on, seed=0):
 
 # ---------------------------------------------------------------------------- oracle (CPU)
 
+def refresh_fraction(wl, seed=0):
+    """Share of (sequence, step) pairs of the workload's denoising steps
+    1..T that refresh, from the oracle's rule (Eq. archer-distance, the age
+    cap) over the workload's own seeded redraws."""
+    from oracle import oracle as O
+    from paper_2608_08086_gb300 import synth
+    B = wl.shape.batch
+    if wl.steps < 1 or B < 1:
+        return 0.0
+    g = synth.traj_initial_tokens(wl, seed)
+    anchor, age = g.copy(), np.zeros(B, np.int32)
+    fired = 0
+    for t in range(1, wl.steps + 1):
+        pos, new = synth.traj_redraw(wl, seed, t, g)
+        g[np.arange(B)[:, None], pos] = new
+        _, flag, anchor, age = O.should_refresh(g, anchor, age, wl.radius_k, wl.max_age)
+        fired += int(flag.sum())
+    return fired / (B * wl.steps)
+
+
 def oracle_sample_step(wl, n_pairs=None, score_rows=8, seed=0):
     """One bounded sample of a step on the fp64 oracle, extrapolated to the full
     step: cached attention of `n_pairs` (sequence, head) pairs of one layer, one
@@ -555,7 +575,7 @@ def oracle_sample_step(wl, n_pairs=None, score_rows=8, seed=0):
         O.decode_scores(z, n_threads=threads)
         t_score = (time.perf_counter() - t0) / score_rows * wl.logits_rows
     pairs = B * Hq
-    q_k = 1.0 / wl.max_age if wl.max_age else 1.0 / 3.0
+    q_k = refresh_fraction(wl, seed)
     per_layer = (1 - q_k) * t_cached_pairs / n_pairs * pairs + q_k * t_refresh_pair * pairs
     step_s = wl.layers * per_layer + t_score
     sample = (f"{n_pairs} (sequence, head) pairs of one cached layer ({G} queries x {P + G} keys, D={D}) and "

@@ -1,0 +1,70 @@
+"""bench.py's host logic, on the CPU: the refresh fraction its CPU baseline
+extrapolates with, the gate that drops a traffic figure once the kernel's
+sources change, the peak table's fallback, and the whole-job rate."""
+import importlib.util
+import json
+import os
+
+import pytest
+
+from paper_2608_08086_gb300 import synth
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def bench():
+    spec = importlib.util.spec_from_file_location("bench_host", os.path.join(ROOT, "bench.py"))
+    mod = importlib.util.module_from_spec(spec)
+    spec.loader.exec_module(mod)
+    return mod
+
+
+def test_refresh_fraction_follows_each_workloads_schedule(bench):
+    # tiny: age cap 4 over 8 steps -> t = 4, 8; the long-prompt GQA workload:
+    # age cap 16 over 32 steps -> t = 16, 32; the 32-layer trajectory: the
+    # distance rule fires every third step (t = 3, 6, ..., 63: 21 of 64)
+    assert bench.refresh_fraction(synth.WORKLOADS["tiny"]) == 2 / 8
+    assert bench.refresh_fraction(synth.WORKLOADS["gqa_long"]) == 2 / 32
+    assert bench.refresh_fraction(synth.WORKLOADS["traj32"]) == 21 / 64
+    # no steps: nothing to refresh
+    assert bench.refresh_fraction(synth.WORKLOADS["llada_layer"]) == 0.0
+
+
+def test_traffic_figure_is_dropped_when_the_sources_change(bench, monkeypatch):
+    key = ("attn_step", "gqa_long")
+    ent = dict(bench.MEASURED_TRAFFIC[key])
+    assert bench.measured_traffic(*key) == ent["bytes"]          # recorded for these sources
+    monkeypatch.setitem(bench.MEASURED_TRAFFIC, key, dict(ent, sha16="0" * 16))
+    assert bench.measured_traffic(*key) is None
+    monkeypatch.setitem(bench.MEASURED_TRAFFIC, key, dict(ent, sources=["no_such_file.cu"]))
+    assert bench.measured_traffic(*key) is None
+    assert bench.measured_traffic("attn_step", "no_such_workload") is None
+
+
+def test_traffic_entries_cover_the_compulsory_bytes(bench):
+    # each recorded DRAM figure is at least what the launch must read:
+    # cached step Q + prompt K/V + response K/V = 209.7 MB (the output write
+    # partly stays in L2); scoring 16 x 512 x 152064 bf16 logits
+    sh = synth.WORKLOADS["gqa_long"].shape
+    reads = 2 * (sh.batch * sh.resp_len * sh.n_heads * sh.head_dim
+                 + 2 * sh.batch * (sh.prompt_len + sh.resp_len) * sh.n_kv_heads * sh.head_dim)
+    assert reads <= bench.MEASURED_TRAFFIC[("attn_step", "gqa_long")]["bytes"] <= reads + 2 * reads // 7
+    logits = 2 * 16 * 512 * 152064
+    assert logits <= bench.MEASURED_TRAFFIC[("scores", "gqa_long")]["bytes"] <= logits * 1.01
+
+
+def test_peaks_fall_back_without_the_measured_table(bench, monkeypatch, tmp_path):
+    monkeypatch.setattr(bench, "ROOT", str(tmp_path))
+    p, kind = bench.peaks()
+    assert kind == "fallback" and p == bench.PEAKS_FALLBACK
+    with open(os.path.join(tmp_path, "MEASURED_PEAKS.json"), "w") as f:
+        json.dump({"hbm_gbs": 1.0, "bf16_tflops": 2.0, "bf16_tflops_sustained": 3.0}, f)
+    p, kind = bench.peaks()
+    assert kind == "measured" and p["hbm_gbs"] == 1.0
+
+
+def test_whole_job_rate(bench):
+    # 4 replicas x 20 steps in 500 ms -> 160 steps/s
+    assert bench.whole_job_rate(4, 20, 500.0) == pytest.approx(160.0)
+    assert bench.max_over_ranks(12.5, False) == 12.5
