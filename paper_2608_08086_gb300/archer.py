@@ -278,6 +278,9 @@ def archer_decode_scores(logits, max_prob, top1, margin, mask_state=None, cur_to
             raise ValueError(f"{n} must hold {rows} {dt} values")
     if cur_prob is not None and (cur_prob.numel() != rows or cur_prob.dtype != torch.float32):
         raise ValueError("cur_prob must hold rows fp32 values")
+    for t, n in ((mask_state, "mask_state"), (cur_tokens, "cur_tokens")):
+        if t is not None and t.numel() != rows:
+            raise ValueError(f"{n} must hold {rows} values")
     if workspace is None:
         workspace = scores_workspace(rows, vocab, logits.device)
     ws_bytes = 0 if workspace is None else workspace.numel() * workspace.element_size()
@@ -336,6 +339,14 @@ def archer_scatter_rows(src, pos, dst0, dst0_row0=0, dst1=None, dst1_row0=0, str
 
 
 def archer_cache_rewrite(shape: archer_shape, k_src, v_src, k_dst, v_dst, refresh_flags=None, stream=None):
+    """Copy each flagged sequence's prompt K/V [B, P, Hkv, D] (bf16) from src to
+    dst; a None source skips that tensor; see include/archer.h."""
+    want = (shape.batch, shape.prompt_len, shape.n_kv_heads, shape.head_dim)
+    for t, n in ((k_src, "k_src"), (v_src, "v_src"), (k_dst, "k_dst"), (v_dst, "v_dst")):
+        if t is not None:
+            _expect(t, want, n)
+    if refresh_flags is not None:
+        _expect(refresh_flags, (shape.batch,), "refresh_flags")
     bf = torch.bfloat16
     _raise(lib.archer_cache_rewrite(ctypes.byref(shape), _ptr(k_src, bf, "k_src"), _ptr(v_src, bf, "v_src"),
                                     _ptr(k_dst, bf, "k_dst"), _ptr(v_dst, bf, "v_dst"),
@@ -367,6 +378,25 @@ class StepGraph:
         B, G = g_cur.shape
         if B != shape.batch or G != shape.resp_len:
             raise ValueError("g_cur must be [batch, resp_len]")
+        # the graph holds raw addresses: every size is checked here, before capture
+        P, Hq, Hkv, D = shape.prompt_len, shape.n_heads, shape.n_kv_heads, shape.head_dim
+        N = P + G
+        want = {"q_all": (B, N, Hq, D), "q_resp": (B, G, Hq, D), "k_prompt_new": (B, P, Hkv, D),
+                "v_prompt_new": (B, P, Hkv, D), "k_resp": (B, G, Hkv, D), "v_resp": (B, G, Hkv, D),
+                "k_cache": (B, P, Hkv, D), "v_cache": (B, P, Hkv, D), "out_full": (B, N, Hq, D),
+                "out_step": (B, G, Hq, D)}
+        for i, l in enumerate(layers):
+            for name, shp in want.items():
+                _expect(l[name], shp, f"layers[{i}].{name}")
+        for t, n in ((g_anchor, "g_anchor"), (age, "age"), (flag_out, "flag_out"), (dist_out, "dist_out"),
+                     (refresh_count, "refresh_count")):
+            if t is not None:
+                _expect(t, (B, G) if n == "g_anchor" else ((1,) if n == "refresh_count" else (B,)), n)
+        if logits is not None:
+            for t, n in ((max_prob, "max_prob"), (top1, "top1"), (margin, "margin"), (cur_prob, "cur_prob"),
+                         (mask_state, "mask_state"), (cur_tokens, "cur_tokens")):
+                if t is not None and t.numel() != B * G:
+                    raise ValueError(f"{n} must hold {B * G} values")
         self._keep = []            # tensors whose addresses the graph holds
         ios = (archer_layer_io * len(layers))()
         for i, l in enumerate(layers):
