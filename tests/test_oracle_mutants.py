@@ -63,6 +63,15 @@ MUTANTS = [
      "const double* kp = k_new + b * per_seq;\n"
      "    const double* vp = v_new + b * per_seq;"),
     ("anchor_not_updated", "g_anchor[(size_t)b * G + i] = g_cur[(size_t)b * G + i];", "(void)0;"),
+    ("cur_prob_gating_inverted", "if (cur_tokens && !masked &&", "if (cur_tokens && masked &&"),
+    ("margin_from_logits", "margin[r] = p[t1] - (t2 >= 0 ? p[t2] : 0.0);",
+     "margin[r] = zr[t1] - (t2 >= 0 ? zr[t2] : 0.0);"),
+    ("refresh_keeps_old_cache", "if (refresh && k_cache != k_new) {", "if (false) {"),
+    ("cleared_flag_recomputes_prompt_rows", "const int32_t begin = refresh ? 0 : P;", "const int32_t begin = 0;"),
+    ("lse_layout_transposed", "if (lse) lse[((size_t)b * Hq + h) * M + i] = l;",
+     "if (lse) lse[((size_t)b * M + i) * Hq + h] = l;"),
+    ("age_never_grows", "age[b] = (int32_t)age_t;", "age[b] = age[b];"),
+    ("age_not_reset_on_refresh", "age[b] = 0;", "age[b] = (int32_t)age_t;"),
 ]
 
 
