@@ -340,7 +340,8 @@ def archer_scatter_rows(src, pos, dst0, dst0_row0=0, dst1=None, dst1_row0=0, str
 
 def archer_cache_rewrite(shape: archer_shape, k_src, v_src, k_dst, v_dst, refresh_flags=None, stream=None):
     """Copy each flagged sequence's prompt K/V [B, P, Hkv, D] (bf16) from src to
-    dst; a None source skips that tensor; see include/archer.h."""
+    dst (all four tensors required; flags None = every sequence); see
+    include/archer.h."""
     want = (shape.batch, shape.prompt_len, shape.n_kv_heads, shape.head_dim)
     for t, n in ((k_src, "k_src"), (v_src, "v_src"), (k_dst, "k_dst"), (v_dst, "v_dst")):
         if t is not None:

@@ -116,3 +116,36 @@ def test_scatter_rows_arguments_rejected(lib):
     assert f(1, 1, 1, 32, p, p, ctypes.c_void_p(0x10008), 4, 0, None, 0, 0, None) == -1   # misaligned
     assert f(-1, 1, 1, 32, p, p, p, 4, 0, None, 0, 0, None) == -1
     assert f(0, 1, 1, 32, None, None, None, 0, 0, None, 0, 0, None) == 0   # nothing to do
+
+
+def test_refresh_and_cache_rewrite_arguments_rejected(lib):
+    lib.archer_last_error.restype = ctypes.c_char_p
+    p, odd = ctypes.c_void_p(0x10000), ctypes.c_void_p(0x10008)
+    f = lib.archer_prompt_refresh
+    f.argtypes = [ctypes.POINTER(Shape)] + [ctypes.c_void_p] * 11 + [ctypes.c_size_t, ctypes.c_void_p]
+    s = Shape(1, 4, 4, 2, 2, 128, 0.0)
+    assert f(ctypes.byref(s), p, p, p, p, p, p, None, None, p, None, None, 0, None) == -1   # NULL v_cache
+    assert f(ctypes.byref(s), p, p, p, p, p, p, None, p, odd, None, None, 0, None) == -1     # misaligned
+    assert b"aligned" in lib.archer_last_error()
+    bad = Shape(1, 4, 4, 3, 2, 128, 0.0)
+    assert f(ctypes.byref(bad), p, p, p, p, p, p, None, p, p, None, None, 0, None) == -1     # Hq % Hkv
+    assert f(None, p, p, p, p, p, p, None, p, p, None, None, 0, None) == -1                  # NULL shape
+    empty = Shape(0, 4, 4, 2, 2, 128, 0.0)
+    assert f(ctypes.byref(empty), p, p, p, p, p, p, None, p, p, None, None, 0, None) == 0    # empty batch
+    g = lib.archer_cache_rewrite
+    g.argtypes = [ctypes.POINTER(Shape)] + [ctypes.c_void_p] * 6
+    assert g(ctypes.byref(s), p, None, p, p, None, None) == -1                               # NULL v_src
+    assert g(ctypes.byref(s), p, p, odd, p, None, None) == -1                                # misaligned
+    assert g(ctypes.byref(Shape(1, 4, 4, 2, 2, 96, 0.0)), p, p, p, p, None, None) == -2      # D 96
+    assert g(ctypes.byref(Shape(1, 0, 4, 2, 2, 128, 0.0)), None, None, None, None, None, None) == 0  # P 0
+
+
+def test_workspace_queries_of_bad_shapes_are_zero(lib):
+    w = lib.archer_attn_workspace_size
+    w.argtypes = [ctypes.POINTER(Shape), ctypes.c_int]
+    w.restype = ctypes.c_size_t
+    assert w(ctypes.byref(Shape(1, 4, 4, 3, 2, 128, 0.0)), 8) == 0       # Hq % Hkv
+    assert w(ctypes.byref(Shape(1, 4, 4, 2, 2, 128, 0.0)), 0) == 0       # no queries
+    assert w(None, 8) == 0
+    lib.archer_status_string.restype = ctypes.c_char_p
+    assert lib.archer_status_string(12345)                                # any code has a string
