@@ -67,3 +67,63 @@ def test_logits_planted_token():
     z = synth.bf16_bits_to_f64(synth.logits(16, 4096, seed=1, std=2.5, boost_max=6.0))
     assert z.shape == (16, 4096)
     assert abs(z.std() - 2.5) < 0.1
+
+
+def test_workloads_match_the_stated_recipe():
+    # the shapes and schedules of the synthetic workloads (the paper's
+    # code-generation settings: LLaDA-shaped layers, 5 % redraw per step,
+    # refresh by distance K = 65 or by an age cap)
+    W = synth.WORKLOADS
+    want = {
+        "tiny": ((1, 128, 64, 4, 4, 64), 1, 8, 8, synth.K_INFINITE, 4, 1024, 64, "f32"),
+        "llada_layer": ((1, 512, 256, 32, 32, 128), 1, 1, 0, synth.K_INFINITE, 0, 0, 0, "bf16"),
+        "scoring": ((4, 0, 256, 1, 1, 128), 1, 1, 0, synth.K_INFINITE, 0, 126464, 1024, "bf16"),
+        "traj32": ((8, 1024, 512, 32, 32, 128), 32, 64, 26, 65, 8, 126464, 0, "bf16"),
+        "gqa_long": ((16, 4096, 512, 28, 4, 128), 32, 32, 26, synth.K_INFINITE, 16, 152064, 16 * 512, "bf16"),
+    }
+    assert set(W) == set(want)
+    for name, (shape, layers, steps, redraws, K, max_age, vocab, rows, dt) in want.items():
+        w = W[name]
+        sh = w.shape
+        got = (sh.batch, sh.prompt_len, sh.resp_len, sh.n_heads, sh.n_kv_heads, sh.head_dim)
+        assert (got, w.layers, w.steps, w.redraws_per_step, w.radius_k, w.max_age, w.vocab, w.logits_rows,
+                w.logits_dtype) == (shape, layers, steps, redraws, K, max_age, vocab, rows, dt), name
+    # 26 of 512 is 5 % rounded to the nearest position
+    assert round(0.05 * 512) == W["traj32"].redraws_per_step == W["gqa_long"].redraws_per_step
+
+
+def test_mask_state_rate_and_tokens_uniform():
+    m = synth.mask_state(64, 4096, seed=3)
+    assert abs(m.mean() - 0.5) < 0.01
+    g = synth.tokens(64, 4096, 16, seed=3, mask=m)
+    assert np.all(g[m == 1] == synth.MASK_TOKEN)
+    counts = np.bincount(g[m == 0], minlength=16)
+    assert counts.min() > 0.9 * counts.mean() and counts.max() < 1.1 * counts.mean()
+
+
+def test_redraws_are_uniform_over_positions_and_other_tokens():
+    # positions: each of G = 64 picked with probability n / G = 8 / 64
+    hits = np.zeros(64)
+    for step in range(2000):
+        hits[synth.redraw_positions(7, step, 0, 64, 8)] += 1
+    assert abs(hits.mean() / 2000 - 8 / 64) < 1e-12
+    assert hits.min() > 0.85 * hits.mean() and hits.max() < 1.15 * hits.mean()
+    # tokens: uniform over the 9 ids other than the current one
+    cur = np.full(20000, 4, dtype=np.int32)
+    new = synth.redraw_tokens(7, 0, 0, cur, 10)
+    c = np.bincount(new, minlength=10)
+    assert c[4] == 0
+    others = np.delete(c, 4)
+    assert others.min() > 0.9 * others.mean() and others.max() < 1.1 * others.mean()
+
+
+def test_planted_token_boost_is_uniform_up_to_its_maximum():
+    # the planted entry of a row is N(0, std^2) + U(0, boost): with std -> 0
+    # (std 1e-6) the row maximum is that boost, uniform on [0, boost_max)
+    z = synth.logits(20000, 64, seed=2, std=1e-6, boost_max=6.0, dtype="f32").astype(np.float64)
+    top = z.max(axis=1)
+    assert top.max() < 6.0 and top.min() >= 0.0
+    assert abs(top.mean() - 3.0) < 0.05 and abs(top.std() - 6.0 / np.sqrt(12.0)) < 0.05
+    # the planted id is uniform over the vocabulary
+    c = np.bincount(z.argmax(axis=1), minlength=64)
+    assert c.min() > 0.75 * c.mean() and c.max() < 1.25 * c.mean()
