@@ -149,3 +149,22 @@ def test_workspace_queries_of_bad_shapes_are_zero(lib):
     assert w(None, 8) == 0
     lib.archer_status_string.restype = ctypes.c_char_p
     assert lib.archer_status_string(12345)                                # any code has a string
+
+
+def test_no_cpu_path_the_binding_and_smoke_fail_loudly(tmp_path):
+    # the binding refuses to import where its library is missing
+    import importlib.util
+    import shutil
+    src = os.path.join(ROOT, "paper_2608_08086_gb300", "archer.py")
+    shutil.copy(src, tmp_path / "archer.py")
+    spec = importlib.util.spec_from_file_location("archer_without_library", tmp_path / "archer.py")
+    mod = importlib.util.module_from_spec(spec)
+    with pytest.raises(ImportError, match="no CPU fallback"):
+        spec.loader.exec_module(mod)
+    # smoke() on a machine without a GPU raises instead of passing on the CPU
+    import torch
+    if torch.cuda.is_available():
+        pytest.skip("a GPU is present")
+    import __graft_entry__
+    with pytest.raises(RuntimeError, match="cuda:0"):
+        __graft_entry__.smoke()
