@@ -68,3 +68,23 @@ def test_whole_job_rate(bench):
     # 4 replicas x 20 steps in 500 ms -> 160 steps/s
     assert bench.whole_job_rate(4, 20, 500.0) == pytest.approx(160.0)
     assert bench.max_over_ranks(12.5, False) == 12.5
+
+
+def test_profile_summaries_and_traffic_table_name_the_same_build(bench):
+    # each committed ncu summary states the source hash it was captured on;
+    # the bench's traffic table must carry the same figure for the same hash
+    import re
+    pdir = os.path.join(ROOT, "profiles")
+    summaries = {"attn_fwd_gqa_long_step.md": ("attn_step", "gqa_long"),
+                 "decode_scores_bulk_gqa_long.md": ("scores", "gqa_long")}
+    for fn, key in summaries.items():
+        text = open(os.path.join(pdir, fn)).read()
+        sha = re.search(r"sha256 prefix ([0-9a-f]{16})", text).group(1)
+        ent = bench.MEASURED_TRAFFIC[key]
+        assert sha == ent["sha16"], fn
+        digits = re.sub(r"[^0-9]", "", re.search(r"traffic[^|]*\|\s*([0-9,]+) B", text).group(1))
+        assert int(digits) == ent["bytes"], fn
+    # the one-tile summary was captured on the same attention sources
+    text = open(os.path.join(pdir, "attn_fwd_single_llada_layer_step.md")).read()
+    assert re.search(r"sha256 prefix ([0-9a-f]{16})", text).group(1) == \
+        bench.MEASURED_TRAFFIC[("attn_step", "gqa_long")]["sha16"]
