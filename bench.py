@@ -315,21 +315,31 @@ def _attn_pair(sh, dev, runs, flush):
     return res
 
 
-def sweep(args):
-    """Per-configuration measurements (one JSON line each): the LLaDA-shaped
-    layer (B1, 32 = 32 heads, D128, P512, G256), decoder scoring on
-    [4 x 256 x 126464] bf16, and the prompt-length sweep G = 256,
-    P = 128 ... 2048 with LLaDA heads (cached step vs refresh of one layer).
-    "cold" launches follow a 256 MB L2-flushing write; "b2b" is back to back
-    from the host; "graph" is back to back from one captured CUDA graph."""
+def per_config(runs, pk, pk_kind):
+    """Per-configuration measurements: the LLaDA-shaped layer (B1, 32 = 32
+    heads, D128, P512, G256; cached step next to its 768-query refresh),
+    decoder scoring on [4 x 256 x 126464] bf16, and the prompt-length sweep
+    G = 256, P = 128 ... 2048 with LLaDA heads (cached step vs refresh of one
+    layer).  "cold" launches follow a 256 MB L2-flushing write; "b2b" is back
+    to back from the host; "graph" is back to back from one captured CUDA
+    graph (the device-side cost of a layer in a chain).  These kernels are
+    timed alone, so their fractions are of the burst peaks."""
     from paper_2608_08086_gb300 import archer as A
     dev = torch.device("cuda")
-    pk, pk_kind = peaks()
     flush = torch.zeros(64 << 20, dtype=torch.float32, device=dev)     # 256 MB > L2
-    runs = max(args.launches, 20)
+    peak_tf = pk["bf16_tflops"]
+
+    def attn(sh):
+        r = _attn_pair(sh, dev, runs, flush)
+        for k in ("step", "refresh"):
+            r[k]["frac_graph"] = r[k]["tflops_graph"] / peak_tf
+            r[k]["frac_cold"] = r[k]["tflops_cold"] / peak_tf
+        r["refresh_over_step_graph"] = r["refresh"]["graph_us"] / r["step"]["graph_us"]
+        return r
+
+    out = {"peak_tflops": peak_tf, "peak_gbs": pk["hbm_gbs"], "peak_kind": f"burst ({pk_kind})", "runs": runs}
     wl = synth.WORKLOADS["llada_layer"]
-    print(json.dumps({"sweep": "llada_layer", "shape": dataclasses.asdict(wl.shape), "runs": runs,
-                      **_attn_pair(wl.shape, dev, runs, flush)}), flush=True)
+    out["llada_layer"] = {"shape": dataclasses.asdict(wl.shape), **attn(wl.shape)}
     wl = synth.WORKLOADS["scoring"]
     rows = wl.logits_rows
     z = synth.device_logits(rows, wl.vocab, dev, seed=0, std=wl.logits_std, boost_max=wl.logits_boost)
@@ -343,15 +353,54 @@ def sweep(args):
     cold, b2b = _time_launches(fn, runs, flush)
     gr = _time_graph(fn, runs)
     nbytes = rows * wl.vocab * 2
-    print(json.dumps({"sweep": "scoring", "rows": rows, "vocab": wl.vocab, "bytes": nbytes, "cold_us": cold,
-                      "b2b_us": b2b, "graph_us": gr, "gbs_cold": nbytes / cold / 1e3,
-                      "frac_cold": nbytes / cold / 1e3 / pk["hbm_gbs"],
-                      "peak_gbs": pk["hbm_gbs"], "peak_kind": pk_kind}), flush=True)
+    out["scoring"] = {"rows": rows, "vocab": wl.vocab, "bytes": nbytes, "cold_us": cold, "b2b_us": b2b,
+                      "graph_us": gr, "gbs_cold": nbytes / cold / 1e3, "gbs_graph": nbytes / gr / 1e3,
+                      "frac_cold": nbytes / cold / 1e3 / pk["hbm_gbs"], "frac_graph": nbytes / gr / 1e3 / pk["hbm_gbs"]}
+    del z, mp, t1, mg, ws
+    sweep_pts = []
     for P in (128, 256, 512, 1024, 2048):
         sh = synth.AttnShape(1, P, 256, 32, 32, 128)
-        print(json.dumps({"sweep": "prompt_len", "P": P, "G": 256, "runs": runs,
-                          **_attn_pair(sh, dev, runs, flush)}), flush=True)
+        sweep_pts.append({"P": P, "G": 256, **attn(sh)})
+    out["prompt_sweep"] = sweep_pts
+    A.archer_check_device()
+    del flush
+    torch.cuda.empty_cache()
+    return out
+
+
+def sweep(args):
+    """The per-configuration measurements of per_config, one JSON line each."""
+    pk, pk_kind = peaks()
+    res = per_config(max(args.launches, 20), pk, pk_kind)
+    print(json.dumps({"sweep": "llada_layer", "runs": res["runs"], **res["llada_layer"]}), flush=True)
+    print(json.dumps({"sweep": "scoring", **res["scoring"], "peak_gbs": res["peak_gbs"],
+                      "peak_kind": res["peak_kind"]}), flush=True)
+    for pt in res["prompt_sweep"]:
+        print(json.dumps({"sweep": "prompt_len", "runs": res["runs"], **pt}), flush=True)
     return 0
+
+
+def compact_configs(res):
+    """The per-configuration results as they go on the bench line: per
+    attention layer the graph-replayed and cold times (us), TFLOP/s and
+    fraction of the burst bf16 peak, per scoring launch GB/s and fraction of
+    the HBM copy peak."""
+    def attn(r):
+        return {k: {"graph_us": round(r[k]["graph_us"], 2), "cold_us": round(r[k]["cold_us"], 2),
+                    "gflop": round(r[k]["gflop"], 3), "tflops_graph": round(r[k]["tflops_graph"], 1),
+                    "frac_graph": round(r[k]["frac_graph"], 4), "tflops_cold": round(r[k]["tflops_cold"], 1)}
+                for k in ("step", "refresh")} | {"refresh_over_step_graph": round(r["refresh_over_step_graph"], 3),
+                                                 "ideal_ratio_N_over_G": r["ideal_ratio_N_over_G"]}
+    sc = res["scoring"]
+    return {"peak_tflops": res["peak_tflops"], "peak_gbs": res["peak_gbs"], "peak_kind": res["peak_kind"],
+            "timing": "graph = mean of launches replayed from one CUDA graph; cold = median single launch after "
+                      "a 256 MB L2-flushing write",
+            "llada_layer": {"shape": "B1, 32/32 heads, D128, P512, G256", **attn(res["llada_layer"])},
+            "scoring": {"shape": "bf16 [4 x 256 x 126464]", "bytes": sc["bytes"],
+                        "graph_us": round(sc["graph_us"], 2), "cold_us": round(sc["cold_us"], 2),
+                        "gbs_graph": round(sc["gbs_graph"], 1), "frac_graph": round(sc["frac_graph"], 4),
+                        "gbs_cold": round(sc["gbs_cold"], 1), "frac_cold": round(sc["frac_cold"], 4)},
+            "prompt_sweep": [{"P": pt["P"], "G": pt["G"], **attn(pt)} for pt in res["prompt_sweep"]]}
 
 
 def staleness(args):
@@ -584,24 +633,38 @@ def oracle_sample_step(wl, n_pairs=None, score_rows=8, seed=0):
     return step_s, sample, threads
 
 
+def config_of(wl, world):
+    """The workload's configuration as both arms print it."""
+    return {"workload": wl.name, "batch": wl.shape.batch, "prompt_len": wl.shape.prompt_len,
+            "resp_len": wl.shape.resp_len, "n_heads": wl.shape.n_heads, "n_kv_heads": wl.shape.n_kv_heads,
+            "head_dim": wl.shape.head_dim, "layers": wl.layers, "vocab": wl.vocab,
+            "redraws_per_step": wl.redraws_per_step, "max_age": wl.max_age,
+            "radius_k": None if wl.radius_k >= synth.K_INFINITE else wl.radius_k,
+            "parallelism": f"replicas{world}" if world > 1 else "single",
+            "l2": "no flush: inputs larger than L2 (prompt K/V of one layer > 129 MB)"}
+
+
 def reference_arm(args, wl):
+    """The oracle timed as it stands, each step the same bounded sample as the
+    default run's cpu_baseline (one (sequence, head) pair per host thread,
+    8 scoring rows), extrapolated to the whole step."""
     rank = int(os.environ.get("RANK", "0"))
     if rank != 0:
         return 0
     for _ in range(args.warmup):
-        oracle_sample_step(wl, n_pairs=4, score_rows=2)
+        oracle_sample_step(wl)
     times = []
     sample = ""
     threads = 0
     for _ in range(args.steps):
-        s, sample, threads = oracle_sample_step(wl, n_pairs=4, score_rows=2)
+        s, sample, threads = oracle_sample_step(wl)
         times.append(s)
     step_s = statistics.median(times)
     value = 1.0 / step_s
     line = {"impl": "reference", "metric": METRIC, "value": value, "unit": "steps/s", "n_gpus": args.gpus,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": step_s * 1e3, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-            "config": {"workload": wl.name},
+            "config": config_of(wl, 1),
             "cpu_baseline": {"kind": "oracle", "value": value, "unit": "steps/s", "cores": threads,
                              "sample": sample + " per step (extrapolated)"},
             "e2e": {"value": value, "unit": "steps/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
@@ -618,10 +681,12 @@ def main():
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--workload", default="gqa_long", choices=["gqa_long", "traj32", "llada_layer"])
-    ap.add_argument("--eager-steps", type=int, default=4)
+    ap.add_argument("--eager-steps", type=int, default=8)
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu", action="store_true")
     ap.add_argument("--no-secondary", action="store_true")
+    ap.add_argument("--no-configs", action="store_true",
+                    help="skip the per-configuration measurements (LLaDA layer, scoring, prompt sweep)")
     ap.add_argument("--kernel-only", choices=["attn_step", "attn_refresh", "scores"], default=None,
                     help="run only a few launches of one kernel (for profiler captures)")
     ap.add_argument("--launches", type=int, default=3)
@@ -741,6 +806,12 @@ def main():
         del h2, e2, t2
         torch.cuda.empty_cache()
 
+    # ---- the single-layer configurations: the LLaDA-shaped layer, scoring on
+    # [4 x 256 x 126464], the prompt-length sweep (each GPU measures its own)
+    configs = None
+    if not args.no_configs:
+        configs = compact_configs(per_config(20, pk, pk_kind))
+
     # ---- CPU baseline: the oracle on a bounded sample (rank 0, N = 1)
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu:
@@ -752,13 +823,7 @@ def main():
             "metric": METRIC, "value": value, "unit": "steps/s", "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": ms / args.steps, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
-            "config": {"workload": wl.name, "batch": wl.shape.batch, "prompt_len": wl.shape.prompt_len,
-                       "resp_len": wl.shape.resp_len, "n_heads": wl.shape.n_heads, "n_kv_heads": wl.shape.n_kv_heads,
-                       "head_dim": wl.shape.head_dim, "layers": wl.layers, "vocab": wl.vocab,
-                       "redraws_per_step": wl.redraws_per_step, "max_age": wl.max_age,
-                       "radius_k": None if wl.radius_k >= synth.K_INFINITE else wl.radius_k,
-                       "parallelism": f"replicas{world}" if world > 1 else "single",
-                       "l2": "no flush: inputs larger than L2 (prompt K/V of one layer > 129 MB)"},
+            "config": config_of(wl, world),
             "refresh_steps_timed": n_ref,
             "step": "CUDA graph per step, refresh branch on the device",
             "host_driven_steps_per_s": host_value,
@@ -775,6 +840,7 @@ def main():
             "gpu_launches": launches,
             "clocks": {"sm_mhz": clk["sm_mhz"], "sm_max_mhz": clk["sm_max_mhz"], "reasons": clk["reasons"]},
             "secondary": secondary,
+            "configs": configs,
             "cpu_baseline": cpu,
         }
         print(json.dumps(line), flush=True)

@@ -138,7 +138,10 @@ int archer_attn_plan_query(const archer_shape* shape, int op, size_t ws_bytes, i
 /* Scratch bytes that let archer_attn_step / archer_prompt_refresh split the
  * key tiles of a launch over n_queries (= G or N) query rows per sequence:
  * n_split * B * Hq * n_queries * (4 D + 8), n_split chosen from the SM count;
- * 0 when the launch's grid already fills the GPU (or the shape is invalid). */
+ * 0 when the launch's grid already fills the GPU (or the shape is invalid).
+ * The paper defines no such scratch: this sizing query, like the workspace
+ * arguments of the attention calls, is this library's own addition (the
+ * split-KV merge needs fp32 partials, and no call allocates). */
 size_t archer_attn_workspace_size(const archer_shape* shape, int n_queries);
 
 /*
@@ -169,6 +172,10 @@ int archer_decode_scores(int batch, int resp_len, int vocab, int dtype, const vo
                          float* max_prob, int32_t* top1, float* margin, float* cur_prob,
                          void* workspace, size_t ws_bytes, void* stream);
 
+/* Workspace bytes archer_decode_scores needs for rows x vocab logits of
+ * either dtype (sized for fp32, which needs the most).  The workspace pair of
+ * archer_decode_scores and this query are this library's additions to the
+ * scoring operation, so that no call allocates. */
 size_t archer_decode_scores_workspace_size(int rows, int vocab);
 
 /*
@@ -180,11 +187,13 @@ size_t archer_decode_scores_workspace_size(int rows, int vocab);
  * without workspace / ws_bytes.
  *   Scratch: a static device array of ARCHER_NOALLOC_SCRATCH_BYTES (4 MiB),
  *   created when the library is loaded on a device and held by that device
- *   until the process exits.  A call needing more
- *   (archer_decode_scores_workspace_size(rows, vocab) > 4 MiB, e.g. more than
- *   about 13,000 rows of a 152,064-entry bf16 vocabulary) returns
- *   ARCHER_ERR_UNSUPPORTED and launches nothing.
- *   The first call on a device looks up the array's device address (this may
+ *   until the process exits.  A call needs 16 bytes per 32 KB chunk of each
+ *   row (rows * ceil(vocab * element size / 32768) * 16 bytes, none when a
+ *   row is one chunk); one needing more than 4 MiB (for a 152,064-entry
+ *   vocabulary: more than 26,214 rows of bf16 logits, or 13,797 rows of fp32)
+ *   returns ARCHER_ERR_UNSUPPORTED and launches nothing.
+ *   The first call on a device, and the first after that device's context was
+ *   replaced (cudaDeviceReset), looks up the array's device address (this may
  *   load the library's device code on that device); make that first call
  *   before any stream capture.
  *   Every call shares the one array per device (which keeps the last call's
@@ -338,6 +347,15 @@ int archer_step_graph_launch(archer_step_graph* graph, void* stream);
 /* Frees the graph; call it after the graph's last launch has completed.
  * NULL is a no-op. */
 int archer_step_graph_destroy(archer_step_graph* graph);
+
+/* Test hook for failure detection (the paper has no counterpart): with
+ * on != 0, every attention launch that follows withholds its last P V product,
+ * so the softmax warps' bounded wait expires (after about 1e6 SM clocks), the
+ * kernel leaves cleanly with TMEM freed, and archer_check_device reports
+ * ARCHER_ERR_TIMEOUT; the outputs of those launches are undefined.  on == 0
+ * restores normal launches.  Process-wide; returns the previous setting.
+ * No GPU fault, trap or hang is involved: every wait stays bounded. */
+int archer_debug_stall_attention(int on);
 
 /* Reads and clears the device-side error word that kernels set when a
  * bounded wait expires.  Synchronises `stream`.  Returns ARCHER_OK or

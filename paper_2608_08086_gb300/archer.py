@@ -89,6 +89,7 @@ def _load():
     L.archer_decoder_update.argtypes = [i, i, ctypes.c_float, ctypes.c_float, ctypes.c_int32, vp, vp, vp, vp, vp,
                                         vp]
     L.archer_check_device.argtypes = [vp]
+    L.archer_debug_stall_attention.argtypes = [i]
     L.archer_status_string.argtypes = [i]
     L.archer_status_string.restype = ctypes.c_char_p
     L.archer_last_error.argtypes = []
@@ -100,7 +101,7 @@ def _load():
     for name in ("archer_attn_step", "archer_prompt_refresh", "archer_decode_scores", "archer_should_refresh",
                  "archer_cache_rewrite", "archer_check_device", "archer_version", "archer_step_graph_create",
                  "archer_decoder_update", "archer_scatter_rows", "archer_attn_plan_query",
-                 "archer_step_graph_launch", "archer_step_graph_destroy"):
+                 "archer_step_graph_launch", "archer_step_graph_destroy", "archer_debug_stall_attention"):
         getattr(L, name).restype = ctypes.c_int
     return L
 
@@ -356,6 +357,13 @@ def archer_cache_rewrite(shape: archer_shape, k_src, v_src, k_dst, v_dst, refres
 
 def archer_check_device(stream=None):
     _raise(lib.archer_check_device(_stream(stream)))
+
+
+def archer_debug_stall_attention(on: bool) -> bool:
+    """Test hook: attention launches withhold their last P V product while on
+    (their bounded wait expires; archer_check_device reports the timeout).
+    Returns the previous setting."""
+    return bool(lib.archer_debug_stall_attention(int(bool(on))))
 
 
 def archer_version() -> int:

@@ -1066,6 +1066,8 @@ attn_combine_kernel(const float* __restrict__ ws_o, const float2* __restrict__ w
 
 // ------------------------------------------------------------------ host side
 
+std::atomic<int> g_debug_stall{0};   // set by archer_debug_stall_attention
+
 constexpr int kMaxSplit = 16;
 constexpr int kMinSplitTiles = 16;  // fewer key tiles: no split
 
@@ -1185,11 +1187,11 @@ int launch_d(const AttnCall& c, cudaStream_t stream) {
   prm.q_begin_cached = c.q_begin_cached;
   prm.default_refresh = c.default_refresh;
   prm.scale_log2 = c.scale * 1.4426950408889634f;
-  // Test hook (host-set): ARCHER_DEBUG_STALL_ATTENTION=1 withholds the last PV
-  // product, so a bounded wait expires after ~1e6 clocks and the call reports
-  // ARCHER_ERR_TIMEOUT through archer_check_device; the context stays usable.
-  const char* stall = std::getenv("ARCHER_DEBUG_STALL_ATTENTION");
-  prm.debug_skip_last_pv = (stall && stall[0] == '1') ? 1 : 0;
+  // Test hook (archer_debug_stall_attention): the launch withholds the last
+  // PV product, so a bounded wait expires after ~1e6 clocks and the call
+  // reports ARCHER_ERR_TIMEOUT through archer_check_device; the context stays
+  // usable.  One relaxed atomic load per launch.
+  prm.debug_skip_last_pv = g_debug_stall.load(std::memory_order_relaxed);
   prm.wait_limit = prm.debug_skip_last_pv ? 1000000ll : kWaitLimitCycles;
   prm.flags = c.flags;
   prm.out = static_cast<__nv_bfloat16*>(c.out);
@@ -1343,3 +1345,7 @@ int cache_rewrite_launch(int B, size_t bytes_per_seq, const void* k_src, const v
 }
 
 }  // namespace archer
+
+extern "C" int archer_debug_stall_attention(int on) {
+  return archer::g_debug_stall.exchange(on ? 1 : 0, std::memory_order_relaxed);
+}

@@ -20,6 +20,8 @@
 #include <cmath>
 #include <mutex>
 
+#include <cuda.h>
+
 #include "archer_device.cuh"
 #include "archer_internal.h"
 
@@ -484,11 +486,15 @@ int chunks_for(int vocab, int dtype) {
 
 }  // namespace
 
-size_t decode_scores_ws_bytes(int rows, int vocab) {
-  // Sized for fp32 logits, which need twice the chunks of bf16 for one vocabulary.
-  const int chunks = chunks_for(vocab, ARCHER_DTYPE_F32);
+size_t decode_scores_ws_bytes_dtype(int rows, int vocab, int dtype) {
+  const int chunks = chunks_for(vocab, dtype);
   if (chunks <= 1 || rows <= 0) return 0;
   return static_cast<size_t>(rows) * chunks * sizeof(Partial);
+}
+
+size_t decode_scores_ws_bytes(int rows, int vocab) {
+  // Sized for fp32 logits, which need twice the chunks of bf16 for one vocabulary.
+  return decode_scores_ws_bytes_dtype(rows, vocab, ARCHER_DTYPE_F32);
 }
 
 int decode_scores_launch(int rows, int vocab, int dtype, const void* logits, int64_t row_stride,
@@ -498,7 +504,7 @@ int decode_scores_launch(int rows, int vocab, int dtype, const void* logits, int
   const int chunks = chunks_for(vocab, dtype);
   Partial* parts = nullptr;
   if (chunks > 1) {
-    const size_t need = decode_scores_ws_bytes(rows, vocab);
+    const size_t need = decode_scores_ws_bytes_dtype(rows, vocab, dtype);
     if (workspace == nullptr || ws_bytes < need) {
       set_error("decode_scores needs a workspace of %zu bytes (got %zu)", need, ws_bytes);
       return ARCHER_ERR_ARG;
@@ -575,11 +581,47 @@ namespace {
 constexpr size_t kNoAllocScratchBytes = ARCHER_NOALLOC_SCRATCH_BYTES;
 static __device__ __align__(256) unsigned char g_scores_scratch[kNoAllocScratchBytes];
 
-// Device address of g_scores_scratch on the current device.  Host code cannot
-// use the array's name as a device pointer (it is a host-side stand-in), so the
-// address is looked up once per device, with that device current.
+// Device address of g_scores_scratch in the current device's context.  Host
+// code cannot use the array's name as a device pointer (it is a host-side
+// stand-in), so the address is looked up with that device current, once per
+// device and context: it is cached with the context's unique ID
+// (cuCtxGetId), and a new context on that device (after cudaDeviceReset, say)
+// gets a fresh lookup instead of a stale address.
+using CtxGetCurrentFn = CUresult (*)(CUcontext*);
+using CtxGetIdFn = CUresult (*)(CUcontext, unsigned long long*);
+
+template <typename Fn>
+Fn driver_fn(const char* name) {
+  void* ptr = nullptr;
+  cudaDriverEntryPointQueryResult q;
+  if (cudaGetDriverEntryPointByVersion(name, &ptr, 12000, cudaEnableDefault, &q) == cudaSuccess &&
+      q == cudaDriverEntryPointSuccess)
+    return reinterpret_cast<Fn>(ptr);
+  return nullptr;
+}
+
+// The unique ID of the calling thread's current context (0 if none or unknown).
+unsigned long long current_context_id() {
+  static CtxGetCurrentFn get_current = nullptr;
+  static CtxGetIdFn get_id = nullptr;
+  static std::once_flag once;
+  std::call_once(once, []() {
+    get_current = driver_fn<CtxGetCurrentFn>("cuCtxGetCurrent");
+    get_id = driver_fn<CtxGetIdFn>("cuCtxGetId");
+  });
+  CUcontext ctx = nullptr;
+  unsigned long long id = 0;
+  if (!get_current || !get_id || get_current(&ctx) != CUDA_SUCCESS || !ctx || get_id(ctx, &id) != CUDA_SUCCESS)
+    return 0;
+  return id;
+}
+
 int scratch_address(void** out) {
-  static void* addr[64] = {nullptr};
+  struct Slot {
+    unsigned long long ctx_id;
+    void* addr;
+  };
+  static Slot slot[64] = {};
   static std::mutex mu;
   int dev = 0;
   cudaError_t e = cudaGetDevice(&dev);
@@ -589,13 +631,15 @@ int scratch_address(void** out) {
     return ARCHER_ERR_UNSUPPORTED;
   }
   std::lock_guard<std::mutex> lock(mu);
-  if (!addr[dev]) {
+  const unsigned long long id = current_context_id();
+  if (!slot[dev].addr || id == 0 || slot[dev].ctx_id != id) {
     void* p = nullptr;
-    e = cudaGetSymbolAddress(&p, g_scores_scratch);
+    e = cudaGetSymbolAddress(&p, g_scores_scratch);      // makes the device's primary context current
     if (e != cudaSuccess) return cuda_status(e, "cudaGetSymbolAddress(scoring scratch)");
-    addr[dev] = p;
+    slot[dev].addr = p;
+    slot[dev].ctx_id = current_context_id();
   }
-  *out = addr[dev];
+  *out = slot[dev].addr;
   return ARCHER_OK;
 }
 
@@ -618,7 +662,11 @@ extern "C" int archer_decode_scores_noalloc(int batch, int resp_len, int vocab, 
     return ARCHER_ERR_UNSUPPORTED;
   }
   if (rows == 0) return ARCHER_OK;
-  const size_t need = decode_scores_ws_bytes(static_cast<int>(rows), vocab);
+  if (dtype != ARCHER_DTYPE_BF16 && dtype != ARCHER_DTYPE_F32) {
+    set_error("dtype %d unsupported", dtype);
+    return ARCHER_ERR_UNSUPPORTED;
+  }
+  const size_t need = decode_scores_ws_bytes_dtype(static_cast<int>(rows), vocab, dtype);
   if (need > kNoAllocScratchBytes) {
     set_error("%lld rows of %d logits need %zu bytes of scoring scratch; the allocation-free entry point has "
               "%zu (use archer_decode_scores with a workspace)",

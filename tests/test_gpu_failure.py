@@ -1,5 +1,6 @@
-"""Failure detection without a GPU fault: a host-set test hook makes the
-attention kernel withhold its last P V product, so the softmax warps' bounded
+"""Failure detection without a GPU fault: a host-set test hook
+(archer_debug_stall_attention) makes the attention kernel withhold its last
+P V product, so the softmax warps' bounded
 wait expires (in both kernel instantiations).  The kernel must leave cleanly (TMEM freed, no trap, no hang),
 archer_check_device must report ARCHER_ERR_TIMEOUT, and the context must stay
 usable: the next call is correct."""
@@ -22,7 +23,7 @@ pytestmark = pytest.mark.gpu
 # whose abort path also ends the walk over its items.
 @pytest.mark.parametrize("B,G,H", [(1, 256, 2), (1, 512, 40), (8, 2560, 8)],
                          ids=["one-tile", "two-tile", "persistent"])
-def test_expired_wait_reports_timeout_and_context_survives(monkeypatch, B, G, H):
+def test_expired_wait_reports_timeout_and_context_survives(B, G, H):
     from paper_2608_08086_gb300 import archer as A
     P, D = 128, 64
     bits = synth.attn_inputs(synth.AttnShape(B, P, G, H, H, D), seed=9)
@@ -31,12 +32,14 @@ def test_expired_wait_reports_timeout_and_context_survives(monkeypatch, B, G, H)
     q = d["q_all"][:, P:].contiguous()
     out = torch.zeros(B, G, H, D, dtype=torch.bfloat16, device="cuda")
     A.archer_check_device()                                  # start from a clean error word
-    monkeypatch.setenv("ARCHER_DEBUG_STALL_ATTENTION", "1")
-    A.archer_attn_step(shape, q, d["k_cache"], d["v_cache"], d["k_resp"], d["v_resp"], out)
+    assert not A.archer_debug_stall_attention(True)
+    try:
+        A.archer_attn_step(shape, q, d["k_cache"], d["v_cache"], d["k_resp"], d["v_resp"], out)
+    finally:
+        assert A.archer_debug_stall_attention(False)
     with pytest.raises(A.ArcherError) as e:
         A.archer_check_device()
     assert e.value.status == A.ARCHER_ERR_TIMEOUT
-    monkeypatch.delenv("ARCHER_DEBUG_STALL_ATTENTION")
     A.archer_check_device()                                  # the word was cleared
     A.archer_attn_step(shape, q, d["k_cache"], d["v_cache"], d["k_resp"], d["v_resp"], out)
     A.archer_check_device()

@@ -331,7 +331,8 @@ def test_scores_full_size_gqa_long_sampled(A):
 
 
 def test_scores_workspace_reuse_is_clean(A):
-    # The ticket counters return to zero: repeated calls give identical results.
+    # The chunk partials in the workspace are rewritten by every call before the
+    # combine kernel reads them: repeated calls give identical results.
     rows, V = 300, 70000
     z = synth.device_logits(rows, V, "cuda", seed=2, std=2.0, boost_max=5.0)
     first = _run_scores(A, z, V)

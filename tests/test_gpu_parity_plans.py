@@ -1,0 +1,196 @@
+"""GPU-vs-oracle parity of every attention launch plan, on inputs that make
+the comparison able to fail.
+
+The workloads' own recipe (Q/K/V drawn N(0,1)/sqrt(D), softmax scale
+1/sqrt(D)) gives scores of standard deviation 1/D: the softmax is nearly
+uniform and every output element is a few thousandths, below the absolute
+tolerance of 2e-2, so a zeroed output or a wrong head would pass.  Here Q, K
+and V are N(0,1) and the scale is 1 (the "sharp" reading of the softmax
+scale): scores of standard deviation sqrt(D), a few keys carry each row, the
+outputs are of order one and the running-max rescale fires across tiles.
+
+Each case pins the plan the call launches (archer_attn_plan_query on this
+GPU): the two-tile kernel (with and without a last wave of single tiles), the
+persistent kernel for the cached step and the refresh (flags absent and
+mixed), and the flat two-tile refresh with flags over a ragged query range.
+Per case:
+  * at least 8 (sequence, head) pairs, chosen from the launch's work items:
+    the first, the last, and items at every depth of the persistent walk
+    (item x runs on CTA x mod SMs as that CTA's (x div SMs)-th item);
+  * every element of at least 64 rows of each pair, always rows 0 and G-1
+    (cached step) or 0, P-1, P and N-1 (refresh), plus tile edges;
+  * out within |gpu - ref| <= 2e-2 + 2e-2 |ref| and lse within
+    1e-3 + 1e-3 |ref| of the fp64 oracle (Sec. 4.1 Eq. archer-attention, Sec.
+    4.2 Algorithm 1 FullForward);
+  * the test can fail: max |ref| >= 0.25, and both a zeroed output and another
+    head's output fail the same comparison;
+  * refresh: untouched rows of a cleared-flag sequence keep their sentinel,
+    and the cache holds the fresh prompt K/V exactly where the flag is set.
+"""
+import zlib
+
+import numpy as np
+import pytest
+import torch
+
+from oracle import oracle as O
+from paper_2608_08086_gb300 import synth
+
+pytestmark = pytest.mark.gpu
+
+ATOL = RTOL = 2e-2
+LSE_TOL = 1e-3
+SENTINEL = 3.0
+
+STEP, REFRESH_ALL, REFRESH_FLAGS = 0, 1, 2
+
+# id: (B, P, G, Hq, Hkv, D), op, flags, expected kernel name, expects a single-tile tail
+CASES = {
+    # 2 pairs x 32 heads x 2 = 128 items: one wave of two-tile CTAs
+    "two_tile_step": ((2, 512, 512, 32, 8, 128), STEP, None, "two_tile", False),
+    # 160 items: 152 pair CTAs and a last wave of 2 x 8 single tiles
+    "two_tile_tail_step": ((5, 512, 256, 32, 32, 128), STEP, None, "two_tile", True),
+    # the long-prompt GQA workload's cached step: 896 items, 5.9 per SM
+    "persistent_step_gqa_long": ((16, 4096, 512, 28, 4, 128), STEP, None, "persistent", False),
+    # the 32-layer trajectory's cached step: 512 items, 3.4 per SM
+    "persistent_step_traj32": ((8, 1024, 512, 32, 32, 128), STEP, None, "persistent", False),
+    # head_dim 64: 256 items
+    "persistent_step_d64": ((8, 1024, 512, 16, 4, 64), STEP, None, "persistent", False),
+    # refresh of every sequence: 6 pairs x 32 x 8 = 1536 items
+    "persistent_refresh_all": ((8, 1024, 512, 32, 32, 128), REFRESH_ALL, None, "persistent", False),
+    # mixed flags: cleared sequences take the cached step in the same walk
+    "persistent_refresh_mixed": ((8, 1024, 512, 32, 32, 128), REFRESH_FLAGS, [1, 0, 0, 1, 1, 0, 1, 0],
+                                 "persistent", False),
+    # the long-prompt GQA refresh: 8064 items, 53 per SM
+    "persistent_refresh_gqa_long": ((16, 4096, 512, 28, 4, 128), REFRESH_ALL, None, "persistent", False),
+    # P = 1000: a refreshed range of 1512 rows is not whole tile pairs, so the
+    # flat two-tile grid runs (768 items, a tail of 2 x 8 single tiles that
+    # falls on the last, refreshed, sequence, with its 104-row last tile)
+    "two_tile_refresh_flags_ragged": ((4, 1000, 512, 32, 8, 128), REFRESH_FLAGS, [0, 1, 0, 1], "two_tile", True),
+}
+
+
+@pytest.fixture(scope="module")
+def A():
+    if not torch.cuda.is_available():
+        pytest.fail("the gpu tests need a CUDA device")
+    from paper_2608_08086_gb300 import archer
+    return archer
+
+
+def host_f64(t):
+    if t.dtype == torch.bfloat16:
+        return synth.bf16_bits_to_f64(t.contiguous().view(torch.int16).cpu().numpy().view(np.uint16))
+    return t.double().cpu().numpy()
+
+
+def out_of_tolerance(got, ref):
+    return np.abs(got - ref) > ATOL + RTOL * np.abs(ref)
+
+
+def sampled_pairs(plan, B, Hq, sms, rng, want=10):
+    """(sequence, head) pairs of the work items: the first, the last, and for
+    every depth k of the walk one item x = k * sms + r, r spread over the
+    CTAs; then random items until `want` distinct pairs."""
+    units, tiles_x = plan["work_items"], plan["work_items"] // (B * Hq)
+    items = [0, units - 1]
+    for k in range((units + sms - 1) // sms):
+        items.append(min(units - 1, k * sms + (37 * k + 11) % sms))
+    pairs = []
+
+    def add(x):
+        bh = (int(x) // (tiles_x * Hq), (int(x) // tiles_x) % Hq)
+        if bh not in pairs:
+            pairs.append(bh)
+
+    for x in items:
+        add(x)
+    for x in rng.integers(0, units, 256):
+        if len(pairs) >= want:
+            break
+        add(x)
+    return pairs
+
+
+def sampled_rows(lo, hi, fixed, rng, n=64):
+    rows = set(r for r in fixed if lo <= r < hi)
+    for r in (lo, lo + 127, lo + 128, lo + 255, lo + 256, hi - 1):
+        if lo <= r < hi:
+            rows.add(r)
+    while len(rows) < min(n, hi - lo):
+        rows.add(int(rng.integers(lo, hi)))
+    return np.array(sorted(rows))
+
+
+@pytest.mark.parametrize("name", list(CASES))
+def test_attention_plan_parity_sharp(A, name):
+    (B, P, G, Hq, Hkv, D), op, flags, kernel, tail = CASES[name]
+    N = P + G
+    sms = torch.cuda.get_device_properties(0).multi_processor_count
+    shape = A.make_shape(B, P, G, Hq, Hkv, D, 1.0)
+    plan = A.archer_attn_plan_query(shape, op, A.archer_attn_workspace_size(shape, G if op == STEP else N), 0)
+    want_kernel = {"two_tile": A.ARCHER_KERNEL_TWO_TILE, "persistent": A.ARCHER_KERNEL_PERSISTENT}[kernel]
+    if sms == 152:
+        assert plan["kernel"] == want_kernel, plan
+        assert (plan["single_tail"] > 0) == tail, plan
+        assert plan["n_split"] == 1, plan
+    elif plan["kernel"] != want_kernel:
+        pytest.skip(f"{sms} SMs plan {name} onto another kernel")
+
+    sh = synth.AttnShape(B, P, G, Hq, Hkv, D)
+    d = synth.device_attn_inputs(sh, "cuda", seed=31, std=1.0)
+    M = G if op == STEP else N
+    out = torch.full((B, M, Hq, D), SENTINEL, dtype=torch.bfloat16, device="cuda")
+    lse = torch.full((B, Hq, M), SENTINEL, dtype=torch.float32, device="cuda")
+    kc, vc = d["k_cache"].clone(), d["v_cache"].clone()
+    fl = None if flags is None else np.array(flags, dtype=np.uint8)
+    if op == STEP:
+        q = d["q_all"][:, P:].contiguous()
+        A.archer_attn_step(shape, q, kc, vc, d["k_resp"], d["v_resp"], out, lse)
+    else:
+        q = d["q_all"]
+        A.archer_prompt_refresh(shape, q, d["k_prompt"], d["v_prompt"], d["k_resp"], d["v_resp"], out, lse, kc, vc,
+                                refresh_flags=None if fl is None else torch.from_numpy(fl).cuda())
+    torch.cuda.synchronize()
+    A.archer_check_device()
+
+    refreshed = [op != STEP and (fl is None or fl[b] != 0) for b in range(B)]
+    if op != STEP:
+        for b in range(B):   # the cache: fresh prompt K/V where refreshed, else kept bit for bit
+            src_k, src_v = (d["k_prompt"], d["v_prompt"]) if refreshed[b] else (d["k_cache"], d["v_cache"])
+            assert torch.equal(kc[b].view(torch.int16), src_k[b].view(torch.int16)), f"k_cache of sequence {b}"
+            assert torch.equal(vc[b].view(torch.int16), src_v[b].view(torch.int16)), f"v_cache of sequence {b}"
+            if not refreshed[b]:   # rows 0..P-1 of a cleared-flag sequence are left alone
+                assert bool((out[b, :P] == SENTINEL).all()) and bool((lse[b, :, :P] == SENTINEL).all())
+
+    rng = np.random.default_rng(zlib.crc32(name.encode()))
+    pairs = sampled_pairs(plan, B, Hq, sms, rng)
+    assert len(pairs) >= 8
+    max_ref = 0.0
+    for b, h in pairs:
+        kvh = h // (Hq // Hkv)
+        sl = (slice(b, b + 1), slice(None), slice(kvh, kvh + 1))
+        kg, vg = host_f64(d["k_resp"][sl]), host_f64(d["v_resp"][sl])
+        if refreshed[b]:
+            kp, vp = host_f64(d["k_prompt"][sl]), host_f64(d["v_prompt"][sl])
+            rows = sampled_rows(0, N, [0, P - 1, P, N - 1], rng)
+            q_rows = rows
+        else:
+            kp, vp = host_f64(d["k_cache"][sl]), host_f64(d["v_cache"][sl])
+            lo = 0 if op == STEP else P          # the query rows of the cached step within `out`
+            rows = sampled_rows(lo, lo + G, [lo, lo + G - 1], rng)
+            q_rows = rows
+        ref, ref_lse = O.attention(host_f64(q[b:b + 1, q_rows, h:h + 1]), kp, vp, kg, vg, 1.0)
+        got = host_f64(out[b:b + 1, rows, h:h + 1])
+        got_lse = host_f64(lse[b:b + 1, h:h + 1, rows])
+        bad = out_of_tolerance(got, ref)
+        assert not bad.any(), (f"{name} b{b} h{h}: {bad.sum()} of {bad.size} elements out of tolerance, max err "
+                               f"{np.abs(got - ref).max():.3e}")
+        err_lse = np.abs(got_lse - ref_lse)
+        assert (err_lse <= LSE_TOL + LSE_TOL * np.abs(ref_lse)).all(), f"{name} b{b} h{h}: lse err {err_lse.max():.3e}"
+        # the comparison can fail: a zeroed output and another head's output
+        assert out_of_tolerance(np.zeros_like(got), ref).any(), f"{name} b{b} h{h}: zeros would pass"
+        other = host_f64(out[b:b + 1, rows, (h + 1) % Hq:(h + 1) % Hq + 1])
+        assert out_of_tolerance(other, ref).any(), f"{name} b{b} h{h}: head {(h + 1) % Hq}'s output would pass"
+        max_ref = max(max_ref, float(np.abs(ref).max()))
+    assert max_ref >= 0.25, f"{name}: largest |ref| {max_ref:.3f} is too small for the tolerance to discriminate"
