@@ -743,9 +743,9 @@ def main():
     host_value = whole_job_rate(world, args.steps, max_over_ranks(arm["ms"], dist_on))
     ks = kernel_stats(tr)
     L = tr.L
-    # per step: 3 row scatters + rule + refresh condition + L attention + scoring (2)
-    # [+ L cache rewrites on refresh steps]
-    launches = args.steps * (3 + 2 + L + (2 if tr.score else 0)) + n_ref * L
+    # per step: 3 row scatters + rule + refresh condition + L attention + scoring (2);
+    # a refresh rewrites the prompt cache inside its attention launch
+    launches = args.steps * (3 + 2 + L + (2 if tr.score else 0))
     flops_step_launch = 4.0 * tr.B * tr.Hq * tr.G * tr.N * tr.D
     flops_refresh_launch = 4.0 * tr.B * tr.Hq * tr.N * tr.N * tr.D
     att = {}

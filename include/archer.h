@@ -84,8 +84,10 @@ int archer_attn_step(const archer_shape* shape, const void* q_resp, const void* 
  *   k_resp, v_resp [B, G, Hkv, D] bf16
  *   out [B, N, Hq, D] bf16; lse [B, Hq, N] fp32 (may be NULL)
  *   k_cache, v_cache [B, P, Hkv, D] bf16: for a refreshed sequence overwritten
- *     with k_prompt_new / v_prompt_new (no copy when the pointers are equal);
- *     for a sequence whose flag is clear, read as the anchored cache.
+ *     with k_prompt_new / v_prompt_new (no copy when the pointers are equal;
+ *     otherwise the two must not overlap); for a sequence whose flag is clear,
+ *     read as the anchored cache.  The rewrite happens inside the attention
+ *     launch: one kernel per call (plus the split merge, when it splits).
  *   refresh_flags [B] uint8 (device; may be NULL = refresh every sequence).
  *     A sequence whose flag is 0 takes the cached step instead: its rows
  *     P..N-1 of out/lse get Attn(Q_g, [K_cache || K_g], ...), its rows 0..P-1
@@ -261,7 +263,9 @@ int archer_scatter_rows(int n_outer, int batch, int n, size_t row_bytes, const v
 
 /* Bit-exact copy of a refreshed sequence's prompt K/V into the cache
  * (the cache rewrite C_r <- C_p(g_t) of Algorithm 1) for sequences whose flag
- * is set (all when flags is NULL).  src/dst [B, P, Hkv, D] bf16. */
+ * is set (all when flags is NULL).  src/dst [B, P, Hkv, D] bf16.  A standalone
+ * copy for callers that rebuild a cache outside a refresh:
+ * archer_prompt_refresh already rewrites the cache inside its own launch. */
 int archer_cache_rewrite(const archer_shape* shape, const void* k_src, const void* v_src,
                          void* k_dst, void* v_dst, const uint8_t* refresh_flags, void* stream);
 

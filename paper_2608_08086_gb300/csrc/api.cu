@@ -159,13 +159,11 @@ int archer_prompt_refresh(const archer_shape* shape, const void* q_all, const vo
   c.kg = k_resp; c.vg = v_resp;
   c.out = out; c.lse = lse;
   c.ws = workspace; c.ws_bytes = ws_bytes;
-  if ((st = attn_launch(c, s))) return st;
-  if (c.P == 0) return ARCHER_OK;
-  const size_t per_seq = static_cast<size_t>(c.P) * c.Hkv * c.D * 2;
-  const bool copy_k = k_prompt_new != k_cache, copy_v = v_prompt_new != v_cache;
-  if (!copy_k && !copy_v) return ARCHER_OK;
-  return cache_rewrite_launch(c.B, per_seq, copy_k ? k_prompt_new : nullptr, copy_v ? v_prompt_new : nullptr,
-                              copy_k ? k_cache : nullptr, copy_v ? v_cache : nullptr, refresh_flags, s);
+  // The cache rewrite C_r <- C_p(g_t) happens inside the attention launch:
+  // the kernel stores each fresh prompt K/V tile it loads for a refreshed
+  // sequence back to the cache (nothing to do where the buffers coincide).
+  c.rewrite = (k_prompt_new != k_cache ? 1 : 0) | (v_prompt_new != v_cache ? 2 : 0);
+  return attn_launch(c, s);
 }
 
 int archer_attn_plan_query(const archer_shape* shape, int op, size_t ws_bytes, int sm_count,

@@ -39,6 +39,10 @@ struct AttnCall {
   int q_begin_cached;     // first query row of a cached sequence
   void* ws;               // nullable: split-KV workspace (see attn_workspace_bytes)
   size_t ws_bytes;
+  // Fused cache rewrite of refreshed sequences: bit 0 stores the fresh prompt
+  // K (kp_refresh) into kp_cached, bit 1 V into vp_cached.  The two buffers of a
+  // pair must not overlap unless they are the same buffer (then no bit).
+  int rewrite = 0;
 };
 
 int attn_launch(const AttnCall& c, cudaStream_t stream);

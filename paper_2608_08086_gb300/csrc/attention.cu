@@ -86,6 +86,12 @@ struct AttnParams {
   float scale_log2;           // softmax_scale * log2(e)
   long long wait_limit;       // SM clocks a bounded wait may take
   int debug_skip_last_pv;     // test hook: withhold the last PV and its commits
+  // Fused cache rewrite (C_r <- C_p(g_t) of Algorithm 1): bit 0 K, bit 1 V.  In
+  // a refreshed sequence, the CTA (or persistent item) of the first query tile
+  // of query head kvh * (Hq / Hkv) -- every key split of it -- stores each fresh
+  // prompt K / V tile it has loaded into shared memory to the cache (the
+  // tensor maps tmKpC / tmVpC), once the tile has landed.
+  int rewrite;
   const uint8_t* flags;
   __nv_bfloat16* out;
   float* lse;
@@ -228,6 +234,7 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
   const int n_p = (p.P + kBN - 1) / kBN;
   const int n_g = (p.G + kBN - 1) / kBN;
   const int j0 = split * p.tiles_per_split;                        // this CTA's first key tile
+  const int rw = (refresh && tp == 0 && tile_off == 0 && h % (p.Hq / p.Hkv) == 0) ? p.rewrite : 0;
   const int T = min(n_p + n_g, j0 + p.tiles_per_split) - j0;      // and its number of tiles
   if (T <= 0) return;      // the host sizes splits so that none is empty; uniform anyway
   const bool partial = p.n_split > 1;
@@ -305,6 +312,34 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
   if (warp == kWarpProducer) {
     // ------------------------------------------------------------ producer
     // The whole warp runs the loop and waits (warp-uniform); lane 0 issues.
+    //
+    // Fused cache rewrite (rw != 0): pair w's prompt tiles are stored to the
+    // cache as soon as the producer has seen the pair land, one bulk group per
+    // pair; before a pair's slot is loaded again, the group of the pair that
+    // held it has finished reading shared memory (the groups after it are the
+    // pairs stored since: one with two slots, two with three).
+    int stored = 0;            // pairs 0 .. stored - 1 handed to the store engine
+    auto store_upto = [&](int v) {
+      for (; stored <= v; ++stored) {
+        if (!warp_wait(bar_full + 8 * slot_of(stored), static_cast<uint32_t>(use_of(stored)) & 1u, abort, p.err,
+                       p.wait_limit))
+          return false;
+        if (lane0) {
+          fence_proxy_async_smem();
+          const int slot = slot_of(stored);
+          for (int part = stored >= 1 ? 0 : 1; part < (stored < T ? 2 : 1); ++part) {
+            const int jg = j0 + (part == 0 ? stored - 1 : stored);
+            if (jg >= n_p || !(rw & (part == 0 ? 2 : 1))) continue;
+            const uint32_t src = sKV + (2 * slot + part) * L::kTile;
+            for (int c = 0; c < L::kChunks; ++c)
+              tma_store_4d(part == 0 ? &tmVpC : &tmKpC, src + c * kChunkBytes, c * 64, kvh, jg * kBN, b);
+          }
+          bulk_commit_group();
+        }
+        __syncwarp();
+      }
+      return true;
+    };
     // Two-tile kernel: the MMA warp's wait for P_A(j) also covers "pair j+1
     // has landed" (the barrier counts kBM + 1 arrivals): once that pair has
     // landed and phase j-1 is over, so that this arrival cannot count towards
@@ -317,6 +352,7 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
       if (!warp_wait(bar_full + 8 * slot_of(v), static_cast<uint32_t>(use_of(v)) & 1u, abort, p.err,
                      p.wait_limit))
         return false;
+      if (rw && !store_upto(v)) return false;
       if (wait_prev && v >= 2 &&
           !warp_wait(bar_p_full, static_cast<uint32_t>(v - 2) & 1u, abort, p.err, p.wait_limit))
         return false;
@@ -333,6 +369,7 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
       if (!warp_wait(bar_full + 8 * slot_of(v), static_cast<uint32_t>(use_of(v)) & 1u, abort, p.err,
                      p.wait_limit))
         return false;
+      if (rw && !store_upto(v)) return false;
       if (j >= 2 &&
           !warp_wait(bar_p_full + 8 * (j & 1), static_cast<uint32_t>((j - 2) >> 1) & 1u, abort, p.err, p.wait_limit))
         return false;
@@ -354,6 +391,11 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
           break;
         if (!(ok = landed(u - 1, false))) break;   // u >= 2: pairs 0 .. u-1 are issued
       } else {
+        // S(0) announced (buffer 0's first completion), polled before the
+        // arrival that lets key step 0 complete that buffer again: the poll
+        // for pair 4 below then waits on the completion right after one this
+        // warp has seen, so its parity cannot alias.
+        if (u == 3 && !(ok = warp_wait(bar_s_full, 0u, abort, p.err, p.wait_limit))) break;
         while (ok && next_j < T && min(next_j + 2, T) <= u - 1) ok = landed1(next_j++);
         if (!ok) break;
         // Slot of pair u free: its previous pair u-3 was last read by P V of
@@ -364,6 +406,10 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
                                   p.err, p.wait_limit))
           break;
       }
+      if (rw && lane0) {       // the stores of the pair that held this slot have read it
+        if constexpr (kSingle) bulk_wait_group_read<2>();
+        else bulk_wait_group_read<1>();
+      }
       if (lane0) issue_pair(u);
       __syncwarp();
     }
@@ -373,6 +419,10 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
       else
         while (ok && next_j < T) ok = landed1(next_j++);
     }
+    // The cache writes are complete before the CTA's shared memory is released
+    // (they depend on no other warp, so this cannot hang).
+    if (rw && lane0) bulk_wait_group_all();
+    __syncwarp();
   } else if (warp == kWarpMma) {
     // ------------------------------------------------------------ MMA issuer
     // Lane 0 runs the schedule alone: its waits are single-thread bounded
@@ -704,7 +754,6 @@ attn_fwd_persist_kernel(const __grid_constant__ CUtensorMap tmQ,
   const uint32_t bar_drain = base + L::kOffDrain;
   const uint32_t bar_o_ready = bar_drain + 8;                    // + 8 * tile: O final for the item
   const uint32_t bar_o_free = bar_o_ready + 16;                  // + 8 * tile: O read by the epilogue
-  const uint32_t bar_q_free = bar_o_free + 16;                   // the item's last Q K^T batch done
   uint32_t* holder = reinterpret_cast<uint32_t*>(gbase + L::kOffHolder);
   volatile int* abort = reinterpret_cast<volatile int*>(gbase + L::kOffAbort);
 
@@ -713,7 +762,7 @@ attn_fwd_persist_kernel(const __grid_constant__ CUtensorMap tmQ,
   auto slot_of = [](int g) { return g & 1; };
   auto phase_of = [](int g) { return static_cast<uint32_t>(g >> 1) & 1u; };
   if (warp == kWarpProducer && lane0) {
-    mbar_init(bar_q_full, 1);
+    mbar_init(bar_q_full, 2);                                    // the Q loads' arrival + the producer's gate
     for (int s = 0; s < L::kSlots; ++s) mbar_init(bar_full + 8 * s, 1);
     for (int i = 0; i < 2; ++i) {
       mbar_init(bar_s_full + 8 * i, 1);
@@ -721,7 +770,6 @@ attn_fwd_persist_kernel(const __grid_constant__ CUtensorMap tmQ,
       mbar_init(bar_o_ready + 8 * i, 1);
       mbar_init(bar_o_free + 8 * i, kBM);
     }
-    mbar_init(bar_q_free, 1);
     *abort = 0;
     mbar_fence_init();
   }
@@ -738,21 +786,36 @@ attn_fwd_persist_kernel(const __grid_constant__ CUtensorMap tmQ,
 
   int last_pair = -1;          // producer: the last pair (running index) whose loads were issued
   int q_loads = 0;             // producer: Q loads issued
+  bool gate_pending = false;   // producer: the latest Q load still lacks its gate arrival
   bool mma_done = false;
   if (warp == kWarpProducer) {
     // ------------------------------------------------------------ producer
-    // Pairs in running order g = k (T + 1) + u.  Before issuing pair g: its
-    // slot's previous pair g-2 was read by MMAs that S_B's completion g-2
-    // covers (for u = 1 that pair is the previous item's last, read by the
-    // P V whose "O final" commit covers it; S_B is not used there because the
-    // next item's prologue may already have moved it two phases on).  Then
-    // the item's Q tiles (u = 0; the same poll says the previous item's last
-    // Q K^T is done), then the arrival on P_A for pair g-1 (the key step that
-    // reads it may start; the poll just before says the phase before is
-    // over), then the loads.
+    // Pairs in running order g = k (T + 1) + u, pair g in slot g & 1 (after
+    // pair g - 2).  The producer polls S_B for every completion in turn, each
+    // poll before its own signal that the completion after the polled one
+    // needs, so a parity poll can never see a phase two away from the one it
+    // means.  With g0 = k (T + 1):
+    //   u = 0   the item's Q tiles (Q full counts the loads' arrival and a
+    //           gate) and pair g0 (K_0).  Q and the slot were last read by the
+    //           previous item's key step T - 2 (its prologue when T = 1),
+    //           which S_B completion g0 - 2, polled at that item's end, covers.
+    //   u = 1   S_B completion g0 - 1 (the previous item's last key step: its
+    //           P V read pair g0 - 1, whose slot pair g0 + 1 takes); then the
+    //           gate, without which this item's prologue cannot complete S_B.
+    //   u >= 2  S_B completion g - 2 (the prologue or key step u - 3, the last
+    //           reads of pair g - 2); then pair g - 1's arrival on P_A, without
+    //           which key step u - 2 cannot complete S_B.
+    //   end     S_B completion g0 + T - 1 (key step T - 2, or the prologue), then
+    //           the arrival for the item's last pair.
+    // An arrival on P_A must fall in the phase it is meant for: each follows an
+    // S_B completion that the MMA warp committed after waiting for the phase
+    // before.
+    // Fused cache rewrite (rw != 0, see AttnParams::rewrite): an item stores
+    // each pair's prompt tiles once the producer has seen the pair land (one
+    // bulk group per pair); before a slot is loaded again the group of the
+    // pair that held it has finished reading shared memory.
     bool ok = true;
     int k = 0;
-    int g_prev_last = -1;      // running index of the previous issued pair
     for (int x = blockIdx.x; ok && x < n_units; x += stride) {
       int b, h;
       bool refresh;
@@ -761,24 +824,53 @@ attn_fwd_persist_kernel(const __grid_constant__ CUtensorMap tmQ,
       const int kvh = h / (p.Hq / p.Hkv);
       const CUtensorMap* mKp = refresh ? &tmKpR : &tmKpC;
       const CUtensorMap* mVp = refresh ? &tmVpR : &tmVpC;
+      const int g0 = k * (T + 1);
+      const int rw = (refresh && q0 == p.q_begin_refresh && h % (p.Hq / p.Hkv) == 0) ? p.rewrite : 0;
+      int stored = g0;         // pairs g0 .. stored - 1 handed to the store engine
+      auto store_upto = [&](int v) {
+        for (; stored <= v; ++stored) {
+          if (!warp_wait(bar_full + 8 * slot_of(stored), phase_of(stored), abort, p.err, p.wait_limit)) return false;
+          if (lane0) {
+            fence_proxy_async_smem();
+            const int uu = stored - g0;
+            for (int part = uu >= 1 ? 0 : 1; part < (uu < T ? 2 : 1); ++part) {
+              const int j = part == 0 ? uu - 1 : uu;
+              if (j >= n_p || !(rw & (part == 0 ? 2 : 1))) continue;
+              const uint32_t src = sKV + (2 * slot_of(stored) + part) * L::kTile;
+              for (int c = 0; c < L::kChunks; ++c)
+                tma_store_4d(part == 0 ? &tmVpC : &tmKpC, src + c * kChunkBytes, c * 64, kvh, j * kBN, b);
+            }
+            bulk_commit_group();
+          }
+          __syncwarp();
+        }
+        return true;
+      };
+      // pair v landed -> its stores (rw) and its arrival on P_A
+      auto arrive_landed = [&](int v) {
+        if (!warp_wait(bar_full + 8 * slot_of(v), phase_of(v), abort, p.err, p.wait_limit)) return false;
+        if (rw && !store_upto(v)) return false;
+        if (lane0) mbar_arrive(bar_p_full);
+        __syncwarp();
+        return true;
+      };
       for (int u = 0; u <= T; ++u) {
-        const int g = k * (T + 1) + u;
-        if (u == 0) {
-          // the previous item's Q K^T batches are done: Q and pair g-2's slot are free
-          if (k >= 1 && !warp_wait(bar_q_free, static_cast<uint32_t>(k - 1) & 1u, abort, p.err, p.wait_limit)) {
+        const int g = g0 + u;
+        if (u == 1) {
+          if (k >= 1 && !warp_wait(bar_s_full + 8, static_cast<uint32_t>(g0 - 1) & 1u, abort, p.err, p.wait_limit)) {
             ok = false;
             break;
           }
-        } else if (u == 1) {
-          if (k >= 1 && !warp_wait(bar_o_ready + 8, static_cast<uint32_t>(k - 1) & 1u, abort, p.err, p.wait_limit)) {
+          if (lane0) mbar_arrive(bar_q_full);                  // the gate
+          __syncwarp();
+          gate_pending = false;
+        } else if (u >= 2) {
+          if (!warp_wait(bar_s_full + 8, static_cast<uint32_t>(g - 2) & 1u, abort, p.err, p.wait_limit) ||
+              !arrive_landed(g - 1)) {
             ok = false;
             break;
           }
-        } else {
-          if (!warp_wait(bar_s_full + 8, static_cast<uint32_t>(g - 2) & 1u, abort, p.err, p.wait_limit)) {
-            ok = false;
-            break;
-          }
+          if (rw && lane0) bulk_wait_group_read<1>();            // pair g - 2's stores have read its slot
         }
         if (u == 0) {
           if (lane0) {
@@ -790,17 +882,7 @@ attn_fwd_persist_kernel(const __grid_constant__ CUtensorMap tmQ,
           }
           __syncwarp();
           ++q_loads;
-        }
-        // pair g-1 landed -> its key step's P_A phase (pairs u = 0 hold K_0
-        // only and are waited by the MMA warp itself; an item's last pair
-        // arrived right after it was issued)
-        if (u >= 2) {
-          if (!warp_wait(bar_full + 8 * slot_of(g_prev_last), phase_of(g_prev_last), abort, p.err, p.wait_limit)) {
-            ok = false;
-            break;
-          }
-          if (lane0) mbar_arrive(bar_p_full);
-          __syncwarp();
+          gate_pending = true;
         }
         if (lane0) {
           const int slot = slot_of(g);
@@ -818,19 +900,21 @@ attn_fwd_persist_kernel(const __grid_constant__ CUtensorMap tmQ,
         }
         __syncwarp();
         last_pair = g;
-        g_prev_last = g;
       }
-      // the item's last pair: its arrival at once, after the phase before it
-      // (no slot poll orders it; the next item's first poll is on "Q free")
-      if (ok && !*abort) {
-        const int pa = k * T + T - 1;                           // its P_A phase
-        ok = warp_wait(bar_full + 8 * slot_of(g_prev_last), phase_of(g_prev_last), abort, p.err, p.wait_limit) &&
-             (pa == 0 || warp_wait(bar_p_full, static_cast<uint32_t>(pa - 1) & 1u, abort, p.err, p.wait_limit));
-        if (ok && lane0) mbar_arrive(bar_p_full);
-        __syncwarp();
+      if (!ok) break;
+      // the item's end: S_B completion g0 + T - 1, then the last pair's arrival
+      if (!warp_wait(bar_s_full + 8, static_cast<uint32_t>(g0 + T - 1) & 1u, abort, p.err, p.wait_limit) ||
+          !arrive_landed(g0 + T)) {
+        ok = false;
+        break;
       }
+      if (rw && lane0) bulk_wait_group_read<0>();   // the next item loads into both slots
+      __syncwarp();
       ++k;
     }
+    // Cache writes complete before the CTA exits (they wait on no other warp).
+    if (lane0) bulk_wait_group_all();
+    __syncwarp();
   } else if (warp == kWarpMma) {
     // ------------------------------------------------------------ MMA issuer
     // Lane 0 alone.  Per item: wait for Q and pair k (T + 1) (K_0), S(0) of
@@ -873,7 +957,6 @@ attn_fwd_persist_kernel(const __grid_constant__ CUtensorMap tmQ,
           issue_qk(t, k_tile_of(g0));
           umma_commit(bar_s_full + 8 * t);
         }
-        if (T == 1) umma_commit(bar_q_free);
         for (int j = 0; ok && j < T; ++j) {
           const bool more = j + 1 < T;
           const int g = g0 + j + 1;                             // pair (V_j, K_{j+1})
@@ -891,7 +974,6 @@ attn_fwd_persist_kernel(const __grid_constant__ CUtensorMap tmQ,
             if (more) issue_qk(t, k_tile_of(g));
             umma_commit(bar_s_full + 8 * t);
             if (!more) umma_commit(bar_o_ready + 8 * t);
-            if (t == 1 && j + 2 == T) umma_commit(bar_q_free);     // the item's last Q K^T batch
           }
         }
         ++k;
@@ -1013,6 +1095,8 @@ attn_fwd_persist_kernel(const __grid_constant__ CUtensorMap tmQ,
     tc_fence_after();
     tmem_dealloc(tmem, kTmemCols);
   } else if (warp == kWarpProducer && aborted) {
+    if (gate_pending && lane0) mbar_arrive(bar_q_full);   // the last Q load's phase can then complete
+    __syncwarp();
     if (q_loads > 0) drain_wait(bar_q_full, static_cast<uint32_t>(q_loads - 1) & 1u, p.wait_limit);
     for (int g = max(0, last_pair - 1); g <= last_pair; ++g) drain_wait(bar_full + 8 * slot_of(g), phase_of(g), p.wait_limit);
   }
@@ -1193,6 +1277,7 @@ int launch_d(const AttnCall& c, cudaStream_t stream) {
   // usable.  One relaxed atomic load per launch.
   prm.debug_skip_last_pv = g_debug_stall.load(std::memory_order_relaxed);
   prm.wait_limit = prm.debug_skip_last_pv ? 1000000ll : kWaitLimitCycles;
+  prm.rewrite = c.P > 0 ? c.rewrite : 0;
   prm.flags = c.flags;
   prm.out = static_cast<__nv_bfloat16*>(c.out);
   prm.lse = c.lse;

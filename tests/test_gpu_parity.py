@@ -149,6 +149,31 @@ def test_prompt_refresh_mixed_flags(A):
     np.testing.assert_array_equal(host_f64(vc), rvc)
 
 
+@pytest.mark.parametrize("case", [(1, 300, 100, 2, 1, 128),      # one-tile CTAs
+                                  (2, 640, 256, 32, 8, 128),     # two-tile CTAs
+                                  (8, 512, 512, 16, 4, 64)])     # the persistent kernel
+def test_fused_cache_rewrite_of_one_tensor(A, case):
+    # The refresh writes the cache from inside the attention launch; with the
+    # fresh prompt K already in the cache buffer only V is written back, and
+    # nothing outside the refreshed sequences' prompt rows changes.
+    B, P, G, Hq, Hkv, D = case
+    sh = synth.AttnShape(B, P, G, Hq, Hkv, D)
+    d = synth.device_attn_inputs(sh, "cuda", seed=25)
+    N = P + G
+    shape = A.make_shape(B, P, G, Hq, Hkv, D)
+    flags = torch.tensor([1, 0] * (B // 2) + [1] * (B % 2), dtype=torch.uint8, device="cuda")
+    kp, vc = d["k_prompt"].clone(), d["v_cache"].clone()
+    out = torch.empty(B, N, Hq, D, dtype=torch.bfloat16, device="cuda")
+    A.archer_prompt_refresh(shape, d["q_all"], kp, d["v_prompt"], d["k_resp"], d["v_resp"], out, None, kp, vc,
+                            refresh_flags=flags)
+    torch.cuda.synchronize()
+    A.archer_check_device()
+    assert torch.equal(kp.view(torch.int16), d["k_prompt"].view(torch.int16))
+    for b in range(B):
+        want = d["v_prompt"][b] if flags[b] else d["v_cache"][b]
+        assert torch.equal(vc[b].view(torch.int16), want.view(torch.int16)), f"v_cache of sequence {b}"
+
+
 def test_refresh_every_step_equals_eager_on_gpu(A):
     # Eq. archer-controller: with the cache just rebuilt, the cached step equals
     # the refresh pass's response rows.  Same kernel, same tiles: bit-identical.
