@@ -214,9 +214,10 @@ def kernel_only(args, wl):
             out = torch.empty(B, G, Hq, D, dtype=torch.bfloat16, device=dev)
             fn = lambda: A.archer_attn_step(shape, q, d["k_cache"], d["v_cache"], d["k_resp"], d["v_resp"], out)  # noqa: E731
         else:
+            # the cache is a buffer of its own, as in the trajectory: the launch rewrites it
             out = torch.empty(B, P + G, Hq, D, dtype=torch.bfloat16, device=dev)
             fn = lambda: A.archer_prompt_refresh(shape, d["q_all"], d["k_prompt"], d["v_prompt"], d["k_resp"],  # noqa: E731
-                                                 d["v_resp"], out, None, d["k_prompt"], d["v_prompt"])
+                                                 d["v_resp"], out, None, d["k_cache"], d["v_cache"])
     else:
         rows = wl.logits_rows
         z = synth.device_logits(rows, wl.vocab, dev, seed=0, std=wl.logits_std, boost_max=wl.logits_boost)
