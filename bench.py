@@ -57,9 +57,13 @@ MEASURED_TRAFFIC = {
     # (kernel, workload): DRAM bytes read + written per launch from one ncu capture
     # (dram__bytes_read.sum + dram__bytes_write.sum), valid only while the kernel's
     # sources hash to sha16 (sha256 over the listed files, first 16 hex digits).
-    ("attn_step", "gqa_long"): {"bytes": 244451328, "sha16": "532ef3f9ec98a409",
-                                "sources": ["attention.cu", "archer_device.cuh", "tmem_ldst.cuh"]},
-    ("scores", "gqa_long"): {"bytes": 2496017920, "sha16": "f609be40559ef555",
+    ("attn_step", "gqa_long"): {"bytes": 209838336 + 34735616, "sha16": "3a07ac8987881a3b",
+                                "sources": ["attention_kernels.cuh", "attention_step.cu", "archer_device.cuh",
+                                            "tmem_ldst.cuh"]},
+    ("attn_refresh", "gqa_long"): {"bytes": 812483840 + 619459072, "sha16": "c7ca06229c3d6094",
+                                   "sources": ["attention_kernels.cuh", "attention_rewrite.cu", "archer_device.cuh",
+                                               "tmem_ldst.cuh"]},
+    ("scores", "gqa_long"): {"bytes": 2491544064 + 4941824, "sha16": "2f70226f5d832439",
                              "sources": ["decode_scores.cu", "archer_device.cuh"]},
 }
 
@@ -754,7 +758,8 @@ def main():
     for kind, fl in (("step", flops_step_launch), ("refresh", flops_refresh_launch)):
         if kind in ks:
             k = ks[kind]
-            att[kind] = {"launches": k["count"], "mean_ms": k["mean_ms"], "tflops": fl / (k["mean_ms"] * 1e9)}
+            att[kind] = {"launches": k["count"], "mean_ms": k["mean_ms"], "tflops": fl / (k["mean_ms"] * 1e9),
+                         "traffic": measured_traffic(f"attn_{kind}", wl.name)}
             tot_flops += fl * k["count"]
             tot_ms += k["total_ms"]
     peak_tf = pk["bf16_tflops_sustained"]
@@ -831,7 +836,7 @@ def main():
             "speedup_vs_refresh_every_step": value / eager_value,
             "eager_steps_per_s": eager_value,
             "attention": att,
-            "roofline": {"bound": "tensor", "kernel": "attn_fwd_persist_kernel<128>", "launches": "cached step",
+            "roofline": {"bound": "tensor", "kernel": "attn_fwd_persist_kernel<128, 0> (persistent two-tile, no rewrite)", "launches": "cached step",
                          "flops_per_launch": flops_step_launch, "achieved": achieved, "peak": peak_tf,
                          "unit": "TFLOP/s", "frac": achieved / peak_tf,
                          "traffic": measured_traffic("attn_step", wl.name),

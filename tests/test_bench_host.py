@@ -52,6 +52,14 @@ def test_traffic_entries_cover_the_compulsory_bytes(bench):
     reads = 2 * (sh.batch * sh.resp_len * sh.n_heads * sh.head_dim
                  + 2 * sh.batch * (sh.prompt_len + sh.resp_len) * sh.n_kv_heads * sh.head_dim)
     assert reads <= bench.MEASURED_TRAFFIC[("attn_step", "gqa_long")]["bytes"] <= reads + 2 * reads // 7
+    # refresh: all N query rows and the fresh prompt K/V read, the output and
+    # the cache (the fused rewrite) written; the copy reads the prompt again
+    N = sh.prompt_len + sh.resp_len
+    q_out = 2 * sh.batch * N * sh.n_heads * sh.head_dim
+    kv_p = 2 * 2 * sh.batch * sh.prompt_len * sh.n_kv_heads * sh.head_dim
+    kv_g = 2 * 2 * sh.batch * sh.resp_len * sh.n_kv_heads * sh.head_dim
+    least = q_out + kv_p + kv_g + q_out // 2 + kv_p      # reads, and writes partly still in L2
+    assert least <= bench.MEASURED_TRAFFIC[("attn_refresh", "gqa_long")]["bytes"] <= 2 * q_out + 3 * kv_p + kv_g
     logits = 2 * 16 * 512 * 152064
     assert logits <= bench.MEASURED_TRAFFIC[("scores", "gqa_long")]["bytes"] <= logits * 1.01
 
@@ -78,6 +86,7 @@ def test_profile_summaries_and_traffic_table_name_the_same_build(bench):
     import re
     pdir = os.path.join(ROOT, "profiles")
     summaries = {"attn_fwd_gqa_long_step.md": ("attn_step", "gqa_long"),
+                 "attn_fwd_gqa_long_refresh.md": ("attn_refresh", "gqa_long"),
                  "decode_scores_bulk_gqa_long.md": ("scores", "gqa_long")}
     for fn, key in summaries.items():
         text = open(os.path.join(pdir, fn)).read()
