@@ -98,9 +98,9 @@ bool make_map(CUtensorMap* map, const void* ptr, int B, int L, int H, int D) {
 
 template <int D>
 int launch_d(const AttnCall& c, cudaStream_t stream) {
-  CUtensorMap mq, mkr, mvr, mkc, mvc, mkg, mvg;
+  CUtensorMap mq, mkr, mvr, mkc, mvc, mkg, mvg, mo;
   bool ok = make_map(&mq, c.q, c.B, c.M, c.Hq, D) && make_map(&mkg, c.kg, c.B, c.G, c.Hkv, D) &&
-            make_map(&mvg, c.vg, c.B, c.G, c.Hkv, D);
+            make_map(&mvg, c.vg, c.B, c.G, c.Hkv, D) && make_map(&mo, c.out, c.B, c.M, c.Hq, D);
   if (ok && c.P > 0) {
     ok = make_map(&mkr, c.kp_refresh, c.B, c.P, c.Hkv, D) && make_map(&mvr, c.vp_refresh, c.B, c.P, c.Hkv, D) &&
          make_map(&mkc, c.kp_cached, c.B, c.P, c.Hkv, D) && make_map(&mvc, c.vp_cached, c.B, c.P, c.Hkv, D);
@@ -173,7 +173,7 @@ int launch_d(const AttnCall& c, cudaStream_t stream) {
   la[0].val.programmaticStreamSerializationAllowed = 1;
   lc.attrs = la;
   lc.numAttrs = 1;
-  const CUtensorMap maps[7] = {mq, mkr, mvr, mkc, mvc, mkg, mvg};
+  const CUtensorMap maps[8] = {mq, mkr, mvr, mkc, mvc, mkg, mvg, mo};
   st = rw ? launch_fwd_rewrite(D, pl.kernel, lc, maps, prm) : launch_fwd_plain(D, pl.kernel, lc, maps, prm);
   if (st || pl.n_split == 1) return st;
   // The merge is a programmatic dependent launch: it is scheduled while the

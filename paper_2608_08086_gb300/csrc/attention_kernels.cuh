@@ -144,7 +144,7 @@ struct Layout {
 
 // Launches attn_fwd_kernel / attn_fwd_persist_kernel (kind = kPlanTwoTile,
 // kPlanOneTile or kPlanPersistent) for head_dim D with the tensor maps
-// m = {Q, K_p refresh, V_p refresh, K_p cached, V_p cached, K_g, V_g}; lc
+// m = {Q, K_p refresh, V_p refresh, K_p cached, V_p cached, K_g, V_g, out}; lc
 // carries the grid, stream and attributes (block size and shared memory are
 // set here).  Without the fused cache rewrite: attention_step.cu; with it:
 // attention_rewrite.cu.
@@ -274,13 +274,60 @@ __device__ __forceinline__ void copy_prompt_all(const AttnParams& p, int cta, in
   }
 }
 
+// The output epilogue: O (fp32 in TMEM, this thread's row r of the tile),
+// scaled by inv_l, rounded to bf16 and written into shared memory at `stage`
+// in the 128-byte-swizzled layout of the output tensor map (64-column chunks
+// of kChunkBytes; row r's 16-byte unit u at (u ^ (r mod 8)) * 16 of its
+// 128-byte row), for one TMA store of the tile.  Rows 16 bytes apart in the
+// banks for every 8 consecutive rows: no bank conflicts.
+template <int D>
+__device__ __forceinline__ void stage_o_row(uint32_t t_lane_o, uint32_t stage, int r, float inv_l) {
+#pragma unroll
+  for (int c0 = 0; c0 < D; c0 += 32) {
+    uint32_t o[32];
+    tmem_ld_32(t_lane_o + c0, o);
+    const uint32_t row = stage + (c0 / 64) * kChunkBytes + static_cast<uint32_t>(r) * 128u;
+#pragma unroll
+    for (int v = 0; v < 4; ++v) {
+      const uint32_t unit = static_cast<uint32_t>((c0 % 64) / 8 + v) ^ static_cast<uint32_t>(r & 7);
+      const uint32_t w0 = pack_bf16x2(__uint_as_float(o[8 * v]) * inv_l, __uint_as_float(o[8 * v + 1]) * inv_l);
+      const uint32_t w1 = pack_bf16x2(__uint_as_float(o[8 * v + 2]) * inv_l, __uint_as_float(o[8 * v + 3]) * inv_l);
+      const uint32_t w2 = pack_bf16x2(__uint_as_float(o[8 * v + 4]) * inv_l, __uint_as_float(o[8 * v + 5]) * inv_l);
+      const uint32_t w3 = pack_bf16x2(__uint_as_float(o[8 * v + 6]) * inv_l, __uint_as_float(o[8 * v + 7]) * inv_l);
+      asm volatile("st.shared.v4.b32 [%0], {%1, %2, %3, %4};" ::"r"(row + unit * 16u), "r"(w0), "r"(w1), "r"(w2),
+                   "r"(w3)
+                   : "memory");
+    }
+  }
+}
+
+// The tile's warpgroup (128 threads, named barrier bar_id) has staged its
+// rows: one thread stores the 128 x D tile to rows q0 .. q0 + 127 of head h of
+// sequence b (rows past the tensor's end are not written) and waits until the
+// store has read shared memory (and, with `complete`, until it is done).
+template <int D>
+__device__ __forceinline__ void store_o_tile(const CUtensorMap* map, uint32_t stage, uint32_t bar_id, bool issuer,
+                                             bool write, int h, int q0, int b, bool complete) {
+  fence_proxy_async_smem();
+  named_barrier(bar_id, kBM);
+  if (issuer) {
+    if (write) {
+#pragma unroll
+      for (int c = 0; c < D / 64; ++c) tma_store_4d(map, stage + c * kChunkBytes, c * 64, h, q0, b);
+    }
+    bulk_commit_group();
+    if (complete) bulk_wait_group_all();
+    else bulk_wait_group_read<0>();
+  }
+}
+
 template <int D, bool kSingle, bool kRewrite>
 __global__ void __launch_bounds__(kRewrite ? kThreadsRw : kThreads, 1)
 attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
                 const __grid_constant__ CUtensorMap tmKpR, const __grid_constant__ CUtensorMap tmVpR,
                 const __grid_constant__ CUtensorMap tmKpC, const __grid_constant__ CUtensorMap tmVpC,
                 const __grid_constant__ CUtensorMap tmKg, const __grid_constant__ CUtensorMap tmVg,
-                const AttnParams p) {
+                const __grid_constant__ CUtensorMap tmO, const AttnParams p) {
   using L = Layout<D, kSingle>;
   if constexpr (kRewrite) {
     if (p.copy_ctas > 0 && static_cast<int>(blockIdx.x) >= static_cast<int>(gridDim.x) - p.copy_ctas) {
@@ -631,14 +678,21 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
           tmem_st_16(t_lane + colO + c0, o);
         }
       };
-      // An expired wait sets the abort flag; the warps then run on over stale
-      // TMEM (in bounds) to the epilogue.
+      // An expired wait sets the abort flag; the warp then stops its key steps
+      // (after a failed wait a parity poll of a later phase could pass on a
+      // stale one, and an arrival on P without the producer's would drive
+      // that barrier's pending count below zero) and goes to the epilogue
+      // over stale TMEM (in bounds).
+      bool failed = false;
       for (int j = 0; j < T; ++j) {
         // kSingle: S(j), P(j) in buffer j & 1 (its (j / 2)-th use)
         const uint32_t bar_sj = kSingle ? bar_s_full + 8 * (j & 1) : bar_s;
         const uint32_t bar_pj = kSingle ? bar_p_full + 8 * (j & 1) : bar_ph;
         const uint32_t col_sj = kSingle ? col_s(j & 1) : colS;
-        warp_wait(bar_sj, kSingle ? (j >> 1) & 1 : j & 1, abort, p.err, p.wait_limit);
+        if (!warp_wait(bar_sj, kSingle ? (j >> 1) & 1 : j & 1, abort, p.err, p.wait_limit)) {
+          failed = true;
+          break;
+        }
         tc_fence_after();
         const int jg = j0 + j;
         const int valid = jg < n_p ? min(kBN, p.P - jg * kBN) : min(kBN, p.G - (jg - n_p) * kBN);
@@ -654,8 +708,8 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
           // of tile j-1; the barrier cannot be further ahead: S(j+3) needs
           // this P).
           if constexpr (kSingle)
-            warp_wait(bar_s_full + 8 * ((j + 1) & 1), static_cast<uint32_t>((j + 1) >> 1) & 1u, abort, p.err,
-                      p.wait_limit);
+            failed = !warp_wait(bar_s_full + 8 * ((j + 1) & 1), static_cast<uint32_t>((j + 1) >> 1) & 1u, abort,
+                                p.err, p.wait_limit);
           const float m_new = fmaxf(m_used, tm);
           const float a = ex2_approx(m_used - m_new);
           m_used = m_new;
@@ -686,9 +740,11 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
         l2 = fadd2(l2, fadd2(acc[0], acc[1]));
         tc_fence_before();
         mbar_arrive(bar_pj);
+        if (failed) break;                 // (the one-tile rescale wait expired)
       }
-      bool ok;
-      if constexpr (kSingle) {
+      bool ok = false;
+      if (failed) {
+      } else if constexpr (kSingle) {
         // O final: the commit after P V of tile T-1 (buffer (T+1) & 1, the
         // phase after S(T-1) on that buffer).
         ok = warp_wait(bar_s_full + 8 * ((T + 1) & 1), static_cast<uint32_t>((T + 1) >> 1) & 1u, abort, p.err,
@@ -717,22 +773,12 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
         }
         if (live) p.ws_ml[row] = make_float2(m_used, l_sum);
       } else {
-        const float inv_l = 1.0f / l_sum;
-        __nv_bfloat16* orow = p.out + ((static_cast<size_t>(b) * p.M + q) * p.Hq + h) * D;
-#pragma unroll
-        for (int c0 = 0; c0 < D; c0 += 32) {
-          uint32_t o[32];
-          tmem_ld_32(t_lane + colO + c0, o);
-          uint32_t w[16];
-#pragma unroll
-          for (int k = 0; k < 16; ++k)
-            w[k] = pack_bf16x2(__uint_as_float(o[2 * k]) * inv_l, __uint_as_float(o[2 * k + 1]) * inv_l);
-          if (live) {
-            uint4* dst = reinterpret_cast<uint4*>(orow + c0);
-#pragma unroll
-            for (int v = 0; v < 4; ++v) dst[v] = make_uint4(w[4 * v], w[4 * v + 1], w[4 * v + 2], w[4 * v + 3]);
-          }
-        }
+        // The tile's Q region is free once O is final (its last reader, the
+        // tile's last Q K^T, finished before): the bf16 tile is staged there
+        // and written by one TMA store.
+        stage_o_row<D>(t_lane + colO, sQ + t * L::kTile, r, 1.0f / l_sum);
+        store_o_tile<D>(&tmO, sQ + t * L::kTile, 1u + t, threadIdx.x == 32 * (kWarpSoftmax0 + 4 * t), ok, h,
+                        q0 + t * kBM, b, true);
         if (live && p.lse)
           p.lse[(static_cast<size_t>(b) * p.Hq + h) * p.M + q] = (m_used + log2f(l_sum)) * 0.69314718055994531f;
       }
@@ -778,13 +824,25 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
 // drained" (the tile's softmax warpgroup, after its epilogue has read O); the
 // MMA warp waits for the latter before the next item's first P V.  Used for
 // two-tile launches without splits whose items all hold two tiles.
+// The persistent kernel's shared memory: the two-tile layout, then "O final"
+// and "O drained" per tile and "staged" (40 bytes), the softmax warpgroups'
+// stop decisions (16 bytes), then, 1024-byte aligned, the output staging
+// buffer of one tile.
+template <int D>
+constexpr uint32_t kPersistStopOff = Layout<D, false>::kUsed + 40 + 8;   // 4 ints: stop decisions (tile, parity)
+template <int D>
+constexpr uint32_t kPersistStageOff = (kPersistStopOff<D> + 16 + 1023u) & ~1023u;
+template <int D>
+constexpr uint32_t kPersistSmemBytes = kPersistStageOff<D> + Layout<D, false>::kTile + 1024;
+static_assert(kPersistSmemBytes<128> <= 232448 && kPersistSmemBytes<64> <= 232448, "shared memory budget");
+
 template <int D, bool kRewrite>
 __global__ void __launch_bounds__(kRewrite ? kThreadsRw : kThreads, 1)
 attn_fwd_persist_kernel(const __grid_constant__ CUtensorMap tmQ,
                         const __grid_constant__ CUtensorMap tmKpR, const __grid_constant__ CUtensorMap tmVpR,
                         const __grid_constant__ CUtensorMap tmKpC, const __grid_constant__ CUtensorMap tmVpC,
                         const __grid_constant__ CUtensorMap tmKg, const __grid_constant__ CUtensorMap tmVg,
-                        const AttnParams p) {
+                        const __grid_constant__ CUtensorMap tmO, const AttnParams p) {
   using L = Layout<D, false>;
   extern __shared__ uint8_t smem_raw[];
   if (p.flags) asm volatile("griddepcontrol.wait;" ::: "memory");
@@ -816,6 +874,13 @@ attn_fwd_persist_kernel(const __grid_constant__ CUtensorMap tmQ,
   const uint32_t bar_drain = base + L::kOffDrain;
   const uint32_t bar_o_ready = bar_drain + 8;                    // + 8 * tile: O final for the item
   const uint32_t bar_o_free = bar_o_ready + 16;                  // + 8 * tile: O read by the epilogue
+  // The output tile's staging buffer (the next item's Q is already loading
+  // into the Q tiles when an item's epilogue runs), used by tile A and tile B
+  // of every item in turn: use n = 2 k + t waits for completion n - 1 of
+  // "staged" (the previous user's store has read it) and completes it once
+  // its own store has.
+  const uint32_t bar_staged = bar_o_free + 16;
+  const uint32_t stage = base + kPersistStageOff<D>;
   uint32_t* holder = reinterpret_cast<uint32_t*>(gbase + L::kOffHolder);
   volatile int* abort = reinterpret_cast<volatile int*>(gbase + L::kOffAbort);
 
@@ -832,6 +897,7 @@ attn_fwd_persist_kernel(const __grid_constant__ CUtensorMap tmQ,
       mbar_init(bar_o_ready + 8 * i, 1);
       mbar_init(bar_o_free + 8 * i, kBM);
     }
+    mbar_init(bar_staged, 1);
     *abort = 0;
     mbar_fence_init();
   }
@@ -1049,16 +1115,26 @@ attn_fwd_persist_kernel(const __grid_constant__ CUtensorMap tmQ,
         tmem_st_16(t_lane + colO + c0, o);
       }
     };
+    // After an expired wait a warp stops its key steps (see attn_fwd_kernel)
+    // and goes to the item's epilogue; whether the walk goes on is decided
+    // once per item for the whole warpgroup (the epilogue's named barrier
+    // needs all four warps): its first thread samples the abort flag into
+    // shared memory before that barrier, every thread reads it after.
+    volatile int* stop_flag = reinterpret_cast<volatile int*>(gbase + kPersistStopOff<D>);
     int k = 0;
-    for (int x = blockIdx.x; x < n_units && !*abort; x += stride) {
+    for (int x = blockIdx.x; x < n_units; x += stride) {
       int b, h;
       bool refresh;
       const int q0 = decode(x, b, h, refresh);
       if (q0 >= p.M) continue;
       float m_used = -INFINITY;
       float2 l2 = make_float2(0.f, 0.f);
+      bool failed = false;
       for (int j = 0; j < T; ++j) {
-        warp_wait(bar_s, static_cast<uint32_t>(k * (T + 1) + j) & 1u, abort, p.err, p.wait_limit);
+        if (!warp_wait(bar_s, static_cast<uint32_t>(k * (T + 1) + j) & 1u, abort, p.err, p.wait_limit)) {
+          failed = true;
+          break;
+        }
         tc_fence_after();
         const int valid = j < n_p ? min(kBN, p.P - j * kBN) : min(kBN, p.G - (j - n_p) * kBN);
         float xs[128];
@@ -1095,33 +1171,31 @@ attn_fwd_persist_kernel(const __grid_constant__ CUtensorMap tmQ,
         tc_fence_before();
         mbar_arrive(bar_ph);
       }
-      const bool ok = warp_wait(bar_o_ready + 8 * t, static_cast<uint32_t>(k) & 1u, abort, p.err, p.wait_limit);
+      const bool ok =
+          !failed && warp_wait(bar_o_ready + 8 * t, static_cast<uint32_t>(k) & 1u, abort, p.err, p.wait_limit);
       tc_fence_after();
       const float l_sum = l2.x + l2.y;
       const int q = q0 + t * kBM + r;
       const bool live = ok && q < p.M;
-      const float inv_l = 1.0f / l_sum;
-      __nv_bfloat16* orow = p.out + ((static_cast<size_t>(b) * p.M + q) * p.Hq + h) * D;
-#pragma unroll
-      for (int c0 = 0; c0 < D; c0 += 32) {
-        uint32_t o[32];
-        tmem_ld_32(t_lane + colO + c0, o);
-        uint32_t w[16];
-#pragma unroll
-        for (int kq = 0; kq < 16; ++kq)
-          w[kq] = pack_bf16x2(__uint_as_float(o[2 * kq]) * inv_l, __uint_as_float(o[2 * kq + 1]) * inv_l);
-        if (live) {
-          uint4* dst = reinterpret_cast<uint4*>(orow + c0);
-#pragma unroll
-          for (int v = 0; v < 4; ++v) dst[v] = make_uint4(w[4 * v], w[4 * v + 1], w[4 * v + 2], w[4 * v + 3]);
-        }
-      }
+      const int use = 2 * k + t;                       // this tile's turn on the staging buffer
+      if (use > 0)
+        warp_wait(bar_staged, static_cast<uint32_t>(use - 1) & 1u, abort, p.err, p.wait_limit);
+      stage_o_row<D>(t_lane + colO, stage, r, 1.0f / l_sum);
+      tc_fence_before();
+      mbar_arrive(bar_o_free + 8 * t);                 // O has been read out of TMEM
+      const bool issuer = threadIdx.x == 32 * (kWarpSoftmax0 + 4 * t);
+      volatile int* stop = stop_flag + 2 * t + (k & 1);  // two slots: the next item's cannot overtake a reader
+      if (issuer) *stop = *abort;
+      store_o_tile<D>(&tmO, stage, 1u + t, issuer, ok, h, q0 + t * kBM, b, false);
+      if (issuer) mbar_arrive(bar_staged);
       if (live && p.lse)
         p.lse[(static_cast<size_t>(b) * p.Hq + h) * p.M + q] = (m_used + log2f(l_sum)) * 0.69314718055994531f;
-      tc_fence_before();
-      mbar_arrive(bar_o_free + 8 * t);
       ++k;
+      if (*stop) break;
     }
+    // the output stores are complete before the CTA exits (they wait on no other thread)
+    if (threadIdx.x == 32 * (kWarpSoftmax0 + 4 * t)) bulk_wait_group_all();
+    __syncwarp();
   }
 
   tc_fence_before();
@@ -1205,7 +1279,8 @@ int launch_fwd(int kind, cudaLaunchConfig_t lc, const CUtensorMap* m, const Attn
     set_error("device ordinal %d out of range", dev);
     return ARCHER_ERR_UNSUPPORTED;
   }
-  const int two = (int)Layout<D, false>::kSmemBytes, one = (int)Layout<D, true>::kSmemBytes, pers = two + 40;
+  const int two = (int)Layout<D, false>::kSmemBytes, one = (int)Layout<D, true>::kSmemBytes,
+            pers = (int)kPersistSmemBytes<D>;
   if (!configured[dev].load(std::memory_order_acquire)) {
     cudaError_t e = cudaFuncSetAttribute(attn_fwd_kernel<D, false, kRw>, cudaFuncAttributeMaxDynamicSharedMemorySize, two);
     if (e == cudaSuccess)
@@ -1219,11 +1294,11 @@ int launch_fwd(int kind, cudaLaunchConfig_t lc, const CUtensorMap* m, const Attn
   lc.dynamicSmemBytes = kind == kPlanOneTile ? one : (kind == kPlanPersistent ? pers : two);
   cudaError_t e;
   if (kind == kPlanOneTile)
-    e = cudaLaunchKernelEx(&lc, attn_fwd_kernel<D, true, kRw>, m[0], m[1], m[2], m[3], m[4], m[5], m[6], prm);
+    e = cudaLaunchKernelEx(&lc, attn_fwd_kernel<D, true, kRw>, m[0], m[1], m[2], m[3], m[4], m[5], m[6], m[7], prm);
   else if (kind == kPlanPersistent)
-    e = cudaLaunchKernelEx(&lc, attn_fwd_persist_kernel<D, kRw>, m[0], m[1], m[2], m[3], m[4], m[5], m[6], prm);
+    e = cudaLaunchKernelEx(&lc, attn_fwd_persist_kernel<D, kRw>, m[0], m[1], m[2], m[3], m[4], m[5], m[6], m[7], prm);
   else
-    e = cudaLaunchKernelEx(&lc, attn_fwd_kernel<D, false, kRw>, m[0], m[1], m[2], m[3], m[4], m[5], m[6], prm);
+    e = cudaLaunchKernelEx(&lc, attn_fwd_kernel<D, false, kRw>, m[0], m[1], m[2], m[3], m[4], m[5], m[6], m[7], prm);
   return cuda_status(e, "attention launch");
 }
 
