@@ -57,13 +57,13 @@ MEASURED_TRAFFIC = {
     # (kernel, workload): DRAM bytes read + written per launch from one ncu capture
     # (dram__bytes_read.sum + dram__bytes_write.sum), valid only while the kernel's
     # sources hash to sha16 (sha256 over the listed files, first 16 hex digits).
-    ("attn_step", "gqa_long"): {"bytes": 209838336 + 34735616, "sha16": "3a07ac8987881a3b",
+    ("attn_step", "gqa_long"): {"bytes": 209787904 + 37175552, "sha16": "ddebb17a4bc03cc6",
                                 "sources": ["attention_kernels.cuh", "attention_step.cu", "archer_device.cuh",
                                             "tmem_ldst.cuh"]},
-    ("attn_refresh", "gqa_long"): {"bytes": 812483840 + 619459072, "sha16": "c7ca06229c3d6094",
+    ("attn_refresh", "gqa_long"): {"bytes": 812035328 + 624442368, "sha16": "50805917049cf74a",
                                    "sources": ["attention_kernels.cuh", "attention_rewrite.cu", "archer_device.cuh",
                                                "tmem_ldst.cuh"]},
-    ("scores", "gqa_long"): {"bytes": 2491544064 + 4941824, "sha16": "2f70226f5d832439",
+    ("scores", "gqa_long"): {"bytes": 2491506944 + 4914944, "sha16": "d9373d9f8e00b106",
                              "sources": ["decode_scores.cu", "archer_device.cuh"]},
 }
 
