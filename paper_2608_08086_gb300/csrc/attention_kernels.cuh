@@ -861,6 +861,33 @@ attn_fwd_persist_kernel(const __grid_constant__ CUtensorMap tmQ,
     return (refresh ? p.q_begin_refresh : p.q_begin_cached) + tp * 2 * kBM;
   };
 
+  // The loads an item starts with -- its two Q tiles and the K/V tiles of its
+  // first two pairs (K_0; V_0, K_1) -- prefetched into L2 (a hint) two to five
+  // key steps before the current item ends, the step staggered over the CTAs
+  // (their items end together, so unstaggered prefetches arrive in one burst).
+  // Without it the next item's Q and first pairs, loaded only once the current
+  // item's last key steps are done, reach the SM after its last P V.
+  auto prefetch_item = [&](int x) {
+    if (x >= n_units) return;
+    int b, h;
+    bool refresh;
+    const int q0 = decode(x, b, h, refresh);
+    if (q0 >= p.M) return;
+    const int kvh = h / (p.Hq / p.Hkv);
+    for (int t = 0; t < 2; ++t)
+      if (q0 + t * kBM < p.M)
+        for (int c = 0; c < L::kChunks; ++c) tma_prefetch_4d(&tmQ, c * 64, h, q0 + t * kBM, b);
+    for (int part = 0; part < 3; ++part) {             // K_0, V_0, K_1
+      const int j = part == 2 ? 1 : 0;
+      if (j >= T) break;
+      const bool is_v = part == 1, in_prompt = j < n_p;
+      const int row = in_prompt ? j * kBN : (j - n_p) * kBN;
+      const CUtensorMap* map = in_prompt ? (is_v ? (refresh ? &tmVpR : &tmVpC) : (refresh ? &tmKpR : &tmKpC))
+                                         : (is_v ? &tmVg : &tmKg);
+      for (int c = 0; c < L::kChunks; ++c) tma_prefetch_4d(map, c * 64, kvh, row, b);
+    }
+  };
+
   const uint32_t raw = smem_u32(smem_raw);
   const uint32_t base = (raw + 1023u) & ~1023u;
   uint8_t* gbase = smem_raw + (base - raw);
@@ -998,6 +1025,7 @@ attn_fwd_persist_kernel(const __grid_constant__ CUtensorMap tmQ,
             for (int c = 0; c < L::kChunks; ++c)
               tma_load_4d(dst + c * kChunkBytes, map, bar_full + 8 * slot, c * 64, kvh, row, b);
           }
+          if (u == max(0, T - 2 - (static_cast<int>(blockIdx.x) & 3))) prefetch_item(x + stride);
         }
         __syncwarp();
         last_pair = g;
