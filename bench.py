@@ -57,13 +57,13 @@ MEASURED_TRAFFIC = {
     # (kernel, workload): DRAM bytes read + written per launch from one ncu capture
     # (dram__bytes_read.sum + dram__bytes_write.sum), valid only while the kernel's
     # sources hash to sha16 (sha256 over the listed files, first 16 hex digits).
-    ("attn_step", "gqa_long"): {"bytes": 209787904 + 37175552, "sha16": "ddebb17a4bc03cc6",
+    ("attn_step", "gqa_long"): {"bytes": 209791232 + 37085696, "sha16": "1febb1f8446ec4a2",
                                 "sources": ["attention_kernels.cuh", "attention_step.cu", "archer_device.cuh",
                                             "tmem_ldst.cuh"]},
-    ("attn_refresh", "gqa_long"): {"bytes": 812035328 + 624442368, "sha16": "50805917049cf74a",
+    ("attn_refresh", "gqa_long"): {"bytes": 812606208 + 624160512, "sha16": "12870841bac99ddd",
                                    "sources": ["attention_kernels.cuh", "attention_rewrite.cu", "archer_device.cuh",
                                                "tmem_ldst.cuh"]},
-    ("scores", "gqa_long"): {"bytes": 2491506944 + 4914944, "sha16": "d9373d9f8e00b106",
+    ("scores", "gqa_long"): {"bytes": 2491495424 + 4868096, "sha16": "99cbda7b470f8633",
                              "sources": ["decode_scores.cu", "archer_device.cuh"]},
 }
 
