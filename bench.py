@@ -455,11 +455,15 @@ def staleness(args):
 
 
 def kernel_stats(tr):
-    """Mean durations (ms) and counts of the attention / scoring launches."""
+    """Mean durations (ms) and counts of the attention / scoring launches:
+    each record spans `launches` launches of one kind back to back (a step's
+    layer loop, or one scoring call), and the mean is total time / launches."""
     by = {}
-    for s, e, kind in tr.attn_events:
-        by.setdefault(kind, []).append(s.elapsed_time(e))
-    return {k: {"count": len(v), "mean_ms": sum(v) / len(v), "total_ms": sum(v)} for k, v in by.items()}
+    for s, e, kind, n in tr.attn_events:
+        t = by.setdefault(kind, [0.0, 0])
+        t[0] += s.elapsed_time(e)
+        t[1] += n
+    return {k: {"count": n, "mean_ms": ms / n, "total_ms": ms} for k, (ms, n) in by.items()}
 
 
 # ---------------------------------------------------------------------------- e2e
@@ -741,8 +745,10 @@ def main():
     del arm
     torch.cuda.empty_cache()
     # ---- the same steps driven from the host (flags read back each step), with
-    # CUDA events around every attention and scoring launch: the per-kernel
-    # durations of the roofline
+    # CUDA events around each step's layer loop (its L attention launches back
+    # to back, as in the graph step: an event between two launches would keep
+    # the second from starting while the first ends) and around every scoring
+    # call: the per-kernel durations of the roofline
     arm = run_arm(wl, "archer", args.steps, args.warmup, dist_on, time_attention=True)
     tr = arm["traj"]
     host_value = whole_job_rate(world, args.steps, max_over_ranks(arm["ms"], dist_on))
@@ -837,6 +843,7 @@ def main():
             "eager_steps_per_s": eager_value,
             "attention": att,
             "roofline": {"bound": "tensor", "kernel": "attn_fwd_persist_kernel<128, 0> (persistent two-tile, no rewrite)", "launches": "cached step",
+                         "timing": "CUDA events around each cached step's layer loop (host-driven arm), / its launches",
                          "flops_per_launch": flops_step_launch, "achieved": achieved, "peak": peak_tf,
                          "unit": "TFLOP/s", "frac": achieved / peak_tf,
                          "traffic": measured_traffic("attn_step", wl.name),

@@ -69,7 +69,8 @@ class DeviceTrajectory:
         self._n_refresh_steps = 0
         self.graph = None
         self.t = -1
-        self.attn_events = []          # (start, end, kind) CUDA events around attention launches
+        self.attn_events = []          # (start, end, kind, launches): CUDA events around a step's layer loop
+                                       # (its launches back to back, as in the untimed step) or a scoring call
         self.time_attention = False
         self.layer_ready = None        # optional per-layer CUDA events a refresh layer waits on
         self._alloc()
@@ -144,7 +145,7 @@ class DeviceTrajectory:
             self.ws = A.scores_workspace(rows, V, dev)
 
     # ------------------------------------------------------------------ pieces
-    def _timed(self, kind, fn):
+    def _timed(self, kind, fn, launches=1):
         if not self.time_attention:
             fn()
             return
@@ -152,26 +153,32 @@ class DeviceTrajectory:
         s.record()
         fn()
         e.record()
-        self.attn_events.append((s, e, kind))
+        self.attn_events.append((s, e, kind, launches))
 
     def _forward(self, refresh: bool, flags):
         outs = []
-        for layer in range(self.L):
-            if refresh:
-                if self.layer_ready is not None:
-                    torch.cuda.current_stream().wait_event(self.layer_ready[layer])
-                self._timed("refresh", lambda: A.archer_prompt_refresh(
-                    self.shape, self.q_all[layer], self.k_new[layer], self.v_new[layer], self.k_resp[layer],
-                    self.v_resp[layer], self.out_full, None, self.k_cache[layer], self.v_cache[layer],
-                    refresh_flags=flags))
-                if self.record:
-                    outs.append(self.out_full.clone())
-            else:
-                self._timed("step", lambda: A.archer_attn_step(
-                    self.shape, self.q_resp[layer], self.k_cache[layer], self.v_cache[layer], self.k_resp[layer],
-                    self.v_resp[layer], self.out_step))
-                if self.record:
-                    outs.append(self.out_step.clone())
+
+        def layers():
+            for layer in range(self.L):
+                if refresh:
+                    if self.layer_ready is not None:
+                        torch.cuda.current_stream().wait_event(self.layer_ready[layer])
+                    A.archer_prompt_refresh(
+                        self.shape, self.q_all[layer], self.k_new[layer], self.v_new[layer], self.k_resp[layer],
+                        self.v_resp[layer], self.out_full, None, self.k_cache[layer], self.v_cache[layer],
+                        refresh_flags=flags)
+                    if self.record:
+                        outs.append(self.out_full.clone())
+                else:
+                    A.archer_attn_step(
+                        self.shape, self.q_resp[layer], self.k_cache[layer], self.v_cache[layer], self.k_resp[layer],
+                        self.v_resp[layer], self.out_step)
+                    if self.record:
+                        outs.append(self.out_step.clone())
+
+        # one event pair around the step's L launches: an event between two
+        # launches would keep the second from starting while the first ends
+        self._timed("refresh" if refresh else "step", layers, self.L)
         return outs
 
     def _score(self, t):
