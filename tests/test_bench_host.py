@@ -99,3 +99,24 @@ def test_profile_summaries_and_traffic_table_name_the_same_build(bench):
     text = open(os.path.join(pdir, "attn_fwd_single_llada_layer_step.md")).read()
     assert re.search(r"sha256 prefix ([0-9a-f]{16})", text).group(1) == \
         bench.MEASURED_TRAFFIC[("attn_step", "gqa_long")]["sha16"]
+
+
+def test_kernel_stats_divide_each_record_by_its_launches(bench):
+    """A record spans a step's layer loop (L launches back to back) or one
+    scoring call; the mean is the total time over all launches of a kind."""
+    class Ev:
+        def __init__(self, t):
+            self.t = t
+
+        def elapsed_time(self, end):
+            return end.t - self.t
+
+    class Traj:
+        attn_events = [(Ev(0.0), Ev(32 * 0.35), "step", 32), (Ev(0.0), Ev(32 * 0.37), "step", 32),
+                       (Ev(0.0), Ev(32 * 3.1), "refresh", 32), (Ev(0.0), Ev(0.41), "score", 1),
+                       (Ev(0.0), Ev(0.43), "score", 1)]
+
+    ks = bench.kernel_stats(Traj())
+    assert ks["step"]["count"] == 64 and ks["step"]["mean_ms"] == pytest.approx(0.36)
+    assert ks["refresh"]["count"] == 32 and ks["refresh"]["mean_ms"] == pytest.approx(3.1)
+    assert ks["score"]["count"] == 2 and ks["score"]["total_ms"] == pytest.approx(0.84)
