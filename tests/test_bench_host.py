@@ -95,10 +95,11 @@ def test_profile_summaries_and_traffic_table_name_the_same_build(bench):
         assert sha == ent["sha16"], fn
         digits = re.sub(r"[^0-9]", "", re.search(r"traffic[^|]*\|\s*([0-9,]+) B", text).group(1))
         assert int(digits) == ent["bytes"], fn
-    # the one-tile summary was captured on the same attention sources
-    text = open(os.path.join(pdir, "attn_fwd_single_llada_layer_step.md")).read()
-    assert re.search(r"sha256 prefix ([0-9a-f]{16})", text).group(1) == \
-        bench.MEASURED_TRAFFIC[("attn_step", "gqa_long")]["sha16"]
+    # the one-tile and the 32-layer trajectory's summaries were captured on the same attention sources
+    for fn in ("attn_fwd_single_llada_layer_step.md", "attn_fwd_traj32_step.md"):
+        text = open(os.path.join(pdir, fn)).read()
+        assert re.search(r"sha256 prefix ([0-9a-f]{16})", text).group(1) == \
+            bench.MEASURED_TRAFFIC[("attn_step", "gqa_long")]["sha16"], fn
 
 
 def test_kernel_stats_divide_each_record_by_its_launches(bench):
