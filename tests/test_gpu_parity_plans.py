@@ -56,6 +56,10 @@ CASES = {
     "persistent_step_traj32": ((8, 1024, 512, 32, 32, 128), STEP, None, "persistent", False),
     # head_dim 64: 256 items
     "persistent_step_d64": ((8, 1024, 512, 16, 4, 64), STEP, None, "persistent", False),
+    # P = 1000: the last prompt key tile holds 104 keys (masked in the softmax), 512 items
+    "persistent_step_ragged_keys": ((8, 1000, 512, 32, 8, 128), STEP, None, "persistent", False),
+    # P = 0: response-only attention, 896 items of 4 key tiles
+    "persistent_step_no_prompt": ((16, 0, 512, 28, 4, 128), STEP, None, "persistent", False),
     # refresh of every sequence: 6 pairs x 32 x 8 = 1536 items
     "persistent_refresh_all": ((8, 1024, 512, 32, 32, 128), REFRESH_ALL, None, "persistent", False),
     # mixed flags: cleared sequences take the cached step in the same walk
