@@ -67,6 +67,10 @@ CASES = {
                                  "persistent", False),
     # the long-prompt GQA refresh: 8064 items, 53 per SM
     "persistent_refresh_gqa_long": ((16, 4096, 512, 28, 4, 128), REFRESH_ALL, None, "persistent", False),
+    # P = 1000, G = 536: N = 1536 whole tile pairs (768 items), both key segments
+    # ragged (the last prompt tile 104 keys, the last response tile 24), and
+    # the fused rewrite copies a 104-row last prompt tile
+    "persistent_refresh_ragged_keys": ((4, 1000, 536, 32, 8, 128), REFRESH_ALL, None, "persistent", False),
     # P = 1000: a refreshed range of 1512 rows is not whole tile pairs, so the
     # flat two-tile grid runs (768 items, a tail of 2 x 8 single tiles that
     # falls on the last, refreshed, sequence, with its 104-row last tile)
