@@ -110,7 +110,9 @@ int archer_prompt_refresh(const archer_shape* shape, const void* q_all, const vo
  * query tiles, one or two per work item; the key range of an item split when
  * the grid leaves SMs idle and the workspace suffices (a merge kernel then
  * follows); a persistent grid of sm_count CTAs when items of two whole tiles
- * outnumber the SMs.  Writes *plan (zeros for batch 0); returns ARCHER_OK, or
+ * outnumber the SMs.  A last wave of items at most half full runs as single
+ * tiles (in a persistent walk, one each on its first CTAs after their items).
+ * Writes *plan (zeros for batch 0); returns ARCHER_OK, or
  * ARCHER_ERR_ARG / ARCHER_ERR_UNSUPPORTED for a shape the calls would reject.
  * Sec. 4.1 defines the attention this plans; the plan itself is this
  * library's. */
@@ -131,7 +133,9 @@ typedef struct archer_attn_plan {
   int key_tiles_per_split;   /* 128-key tiles one split walks                     */
   int work_items;            /* items over (sequence, head, query range, split)   */
   int grid;                  /* CTAs of the attention launch                      */
-  int single_tail;           /* trailing one-tile CTAs of a two-tile launch       */
+  int single_tail;           /* last-wave items run as single tiles (a two-tile  */
+                             /* launch: appended one-tile CTAs; persistent: the  */
+                             /* walk's first 2 x this CTAs take one tile each)   */
   size_t split_workspace;    /* workspace bytes a split wants (0: no split wanted) */
 } archer_attn_plan;
 int archer_attn_plan_query(const archer_shape* shape, int op, size_t ws_bytes, int sm_count,

@@ -117,6 +117,10 @@ struct AttnParams {
   int B, tiles_x, n_unit_ctas;
   float* ws_o;                // [n_split, B, Hq, M, D] fp32
   float2* ws_ml;              // [n_split, B, Hq, M] (max in log2 units, row sum)
+  // Persistent kernel: it walks items 0 .. n_unit_ctas - 1 in pairs; with
+  // n_lone > 0 the items after them run as n_lone single query tiles, CTA x <
+  // n_lone taking tile x mod 2 of item n_unit_ctas + x / 2 after its items.
+  int n_lone;
 };
 
 // kSingle: the one-tile kernel (one Q tile, three pair slots, S double
@@ -183,6 +187,13 @@ __device__ __forceinline__ bool warp_wait(uint32_t bar, uint32_t parity, volatil
       return false;
     }
   }
+}
+
+// v, as a value the compiler cannot see through: what is computed from it is
+// recomputed there, not kept alive from an earlier computation of the same.
+__device__ __forceinline__ int opaque_int(int v) {
+  asm volatile("" : "+r"(v));
+  return v;
 }
 
 __device__ __forceinline__ float max3f(float a, float b, float c) {
@@ -826,17 +837,19 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
 // two-tile launches without splits whose items all hold two tiles.
 // The persistent kernel's shared memory: the two-tile layout, then "O final"
 // and "O drained" per tile and "staged" (40 bytes), the softmax warpgroups'
-// stop decisions (16 bytes), then, 1024-byte aligned, the output staging
-// buffer of one tile.
+// stop decisions (16 bytes), the single-tile tail's barriers (64 bytes), then,
+// 1024-byte aligned, the output staging buffer of one tile.
 template <int D>
 constexpr uint32_t kPersistStopOff = Layout<D, false>::kUsed + 40 + 8;   // 4 ints: stop decisions (tile, parity)
 template <int D>
-constexpr uint32_t kPersistStageOff = (kPersistStopOff<D> + 16 + 1023u) & ~1023u;
+constexpr uint32_t kPersistLoneOff = kPersistStopOff<D> + 16;          // 8 barriers of the single-tile tail
+template <int D>
+constexpr uint32_t kPersistStageOff = (kPersistLoneOff<D> + 64 + 1023u) & ~1023u;
 template <int D>
 constexpr uint32_t kPersistSmemBytes = kPersistStageOff<D> + Layout<D, false>::kTile + 1024;
 static_assert(kPersistSmemBytes<128> <= 232448 && kPersistSmemBytes<64> <= 232448, "shared memory budget");
 
-template <int D, bool kRewrite>
+template <int D, bool kRewrite, bool kLone>
 __global__ void __launch_bounds__(kRewrite ? kThreadsRw : kThreads, 1)
 attn_fwd_persist_kernel(const __grid_constant__ CUtensorMap tmQ,
                         const __grid_constant__ CUtensorMap tmKpR, const __grid_constant__ CUtensorMap tmVpR,
@@ -844,11 +857,12 @@ attn_fwd_persist_kernel(const __grid_constant__ CUtensorMap tmQ,
                         const __grid_constant__ CUtensorMap tmKg, const __grid_constant__ CUtensorMap tmVg,
                         const __grid_constant__ CUtensorMap tmO, const AttnParams p) {
   using L = Layout<D, false>;
+  static_assert(!(kRewrite && kLone), "the single-tile tail serves cached steps (no cache rewrite)");
   extern __shared__ uint8_t smem_raw[];
   if (p.flags) asm volatile("griddepcontrol.wait;" ::: "memory");
   asm volatile("griddepcontrol.launch_dependents;");
 
-  const int n_units = p.tiles_x * p.Hq * p.B;
+  const int n_units = kLone ? p.n_unit_ctas : p.tiles_x * p.Hq * p.B;   // items walked in pairs
   const int n_p = (p.P + kBN - 1) / kBN;
   const int n_g = (p.G + kBN - 1) / kBN;
   const int T = n_p + n_g;                                       // key tiles per item (no splits)
@@ -888,6 +902,29 @@ attn_fwd_persist_kernel(const __grid_constant__ CUtensorMap tmQ,
     }
   };
 
+  // The CTA's single tail tile (kLone, blockIdx.x < n_lone): its first query
+  // row (>= M: nothing to do), and the L2 prefetch of its Q tile, K_0, V_0, K_1.
+  auto lone_q0 = [&](int& b, int& h, bool& refresh, int cta = static_cast<int>(blockIdx.x)) {
+    return decode(n_units + cta / 2, b, h, refresh) + (cta & 1) * kBM;
+  };
+  auto prefetch_lone = [&]() {
+    int b, h;
+    bool refresh;
+    const int q0 = lone_q0(b, h, refresh);
+    if (q0 >= p.M) return;
+    const int kvh = h / (p.Hq / p.Hkv);
+    for (int c = 0; c < L::kChunks; ++c) tma_prefetch_4d(&tmQ, c * 64, h, q0, b);
+    for (int part = 0; part < 3; ++part) {             // K_0, V_0, K_1
+      const int j = part == 2 ? 1 : 0;
+      if (j >= T) break;
+      const bool is_v = part == 1, in_prompt = j < n_p;
+      const int row = in_prompt ? j * kBN : (j - n_p) * kBN;
+      const CUtensorMap* map = in_prompt ? (is_v ? (refresh ? &tmVpR : &tmVpC) : (refresh ? &tmKpR : &tmKpC))
+                                         : (is_v ? &tmVg : &tmKg);
+      for (int c = 0; c < L::kChunks; ++c) tma_prefetch_4d(map, c * 64, kvh, row, b);
+    }
+  };
+
   const uint32_t raw = smem_u32(smem_raw);
   const uint32_t base = (raw + 1023u) & ~1023u;
   uint8_t* gbase = smem_raw + (base - raw);
@@ -908,6 +945,18 @@ attn_fwd_persist_kernel(const __grid_constant__ CUtensorMap tmQ,
   // its own store has.
   const uint32_t bar_staged = bar_o_free + 16;
   const uint32_t stage = base + kPersistStageOff<D>;
+  // The single-tile tail (kLone): CTA x < n_lone, after its items, takes tile
+  // x mod 2 of item n_units + x / 2 alone, on the one-tile kernel's schedule
+  // with barriers of its own: Q, two pair slots (pair u = V_{u-2} and K_u in
+  // slot u mod 2), one S barrier per S buffer (S(j) in TMEM buffer j mod 2 --
+  // the S columns of tiles A and B -- committed after Q K_j^T; the commit
+  // after key step j's P V announces S(j + 2) and says that P V is done), one
+  // P barrier per S buffer (P(j) on barrier j mod 2: the warpgroup's 128
+  // threads and the producer's "pair j + 2 landed"; a thread can read S(j + 1)
+  // before P(j) is complete, never S(j + 2), so its arrivals never run two
+  // steps ahead on one barrier) and O final.
+  const uint32_t lone = base + kPersistLoneOff<D>;
+  const uint32_t lq_full = lone, l_full = lone + 8, l_s = lone + 24, l_p = lone + 40, l_o = lone + 56;
   uint32_t* holder = reinterpret_cast<uint32_t*>(gbase + L::kOffHolder);
   volatile int* abort = reinterpret_cast<volatile int*>(gbase + L::kOffAbort);
 
@@ -925,6 +974,15 @@ attn_fwd_persist_kernel(const __grid_constant__ CUtensorMap tmQ,
       mbar_init(bar_o_free + 8 * i, kBM);
     }
     mbar_init(bar_staged, 1);
+    if constexpr (kLone) {
+      mbar_init(lq_full, 1);
+      for (int i = 0; i < 2; ++i) {
+        mbar_init(l_full + 8 * i, 1);
+        mbar_init(l_s + 8 * i, 1);
+        mbar_init(l_p + 8 * i, kBM + 1);
+      }
+      mbar_init(l_o, 1);
+    }
     *abort = 0;
     mbar_fence_init();
   }
@@ -941,6 +999,8 @@ attn_fwd_persist_kernel(const __grid_constant__ CUtensorMap tmQ,
 
   int last_pair = -1;          // producer: the last pair (running index) whose loads were issued
   int q_loads = 0;             // producer: Q loads issued
+  int lone_use0 = -1, lone_use1 = -1;   // producer: the single tail tile's latest use of pair slot 0 / 1
+  bool lone_q = false;         // producer: the single tail tile's Q load issued
   bool gate_pending = false;   // producer: the latest Q load still lacks its gate arrival
   bool mma_done = false;
   if (warp == kWarpProducer) {
@@ -1025,7 +1085,14 @@ attn_fwd_persist_kernel(const __grid_constant__ CUtensorMap tmQ,
             for (int c = 0; c < L::kChunks; ++c)
               tma_load_4d(dst + c * kChunkBytes, map, bar_full + 8 * slot, c * 64, kvh, row, b);
           }
-          if (u == max(0, T - 2 - (static_cast<int>(blockIdx.x) & 3))) prefetch_item(x + stride);
+          if (u == max(0, T - 2 - (static_cast<int>(blockIdx.x) & 3))) {
+            if constexpr (kLone) {
+              if (x + stride < n_units) prefetch_item(x + stride);
+              else if (static_cast<int>(blockIdx.x) < p.n_lone) prefetch_lone();
+            } else {
+              prefetch_item(x + stride);
+            }
+          }
         }
         __syncwarp();
         last_pair = g;
@@ -1038,6 +1105,71 @@ attn_fwd_persist_kernel(const __grid_constant__ CUtensorMap tmQ,
         break;
       }
       ++k;
+    }
+    if constexpr (kLone) {
+      // ------------------------------------------------ the single tail tile
+      // Its Q tile and first pair wait for S_B completion k (T + 1) - 1, the
+      // last item's last key step (its P V read both pair slots; Q was last
+      // read by key step T - 2, polled at that item's end), the next S_B
+      // completion in turn.  Pair u (V_{u-2}, K_u) goes into slot u mod 2 once
+      // the commit announcing S(u - 2) -- completion u / 2 - 1 of that S
+      // buffer's barrier, after the last reads of pair u - 2 -- is seen.  Once
+      // the pair has landed the producer arrives on P(u - 2)'s barrier: the
+      // commit it polled followed the MMA warp's wait for that barrier's
+      // previous phase (P(u - 4)), so the arrival falls in its own phase.
+      // Each poll comes before the producer's own arrival that the next
+      // completion of its barrier needs.
+      int b = 0, h = 0;
+      bool refresh = false;
+      const int q0 = static_cast<int>(blockIdx.x) < p.n_lone ? lone_q0(b, h, refresh) : p.M;   // decoded only if it exists
+      if (ok && q0 < p.M) {
+        const int kvh = h / (p.Hq / p.Hkv);
+        const CUtensorMap* mKp = refresh ? &tmKpR : &tmKpC;
+        const CUtensorMap* mVp = refresh ? &tmVpR : &tmVpC;
+        ok = k == 0 ||
+             warp_wait(bar_s_full + 8, static_cast<uint32_t>(k * (T + 1) - 1) & 1u, abort, p.err, p.wait_limit);
+        if (ok) {
+          if (lane0) {
+            mbar_arrive_expect_tx(lq_full, L::kTile);
+            for (int c = 0; c < L::kChunks; ++c) tma_load_4d(sQ + c * kChunkBytes, &tmQ, lq_full, c * 64, h, q0, b);
+          }
+          __syncwarp();
+          lone_q = true;
+        }
+        for (int u = 0; ok && u <= T + 1; ++u) {
+          if (u == 1 && T < 2) continue;                   // no K_1
+          const int slot = u & 1;
+          if (u >= 2 &&
+              !warp_wait(l_s + 8 * slot, static_cast<uint32_t>(u / 2 - 1) & 1u, abort, p.err, p.wait_limit)) {
+            ok = false;
+            break;
+          }
+          if (lane0) {
+            const bool has_v = u >= 2, has_k = u < T;
+            mbar_arrive_expect_tx(l_full + 8 * slot, (has_v && has_k ? 2 : 1) * L::kTile);
+            for (int part = has_v ? 0 : 1; part < (has_k ? 2 : 1); ++part) {
+              const int j = part == 0 ? u - 2 : u;         // key tile
+              const bool in_prompt = j < n_p;
+              const int row = in_prompt ? j * kBN : (j - n_p) * kBN;
+              const CUtensorMap* map = in_prompt ? (part == 0 ? mVp : mKp) : (part == 0 ? &tmVg : &tmKg);
+              const uint32_t dst = sKV + (2 * slot + part) * L::kTile;
+              for (int c = 0; c < L::kChunks; ++c)
+                tma_load_4d(dst + c * kChunkBytes, map, l_full + 8 * slot, c * 64, kvh, row, b);
+            }
+          }
+          __syncwarp();
+          if (slot) lone_use1 = u >> 1;
+          else lone_use0 = u >> 1;
+          if (u >= 2) {
+            if (!warp_wait(l_full + 8 * slot, static_cast<uint32_t>(u >> 1) & 1u, abort, p.err, p.wait_limit)) {
+              ok = false;
+              break;
+            }
+            if (lane0) mbar_arrive(l_p + 8 * slot);      // P(u - 2): barrier (u - 2) mod 2 = slot
+            __syncwarp();
+          }
+        }
+      }
     }
     __syncwarp();              // reconverged before the teardown
   } else if (warp >= kWarpCopy) {        // present only in the kRewrite kernels (11 warps)
@@ -1117,6 +1249,61 @@ attn_fwd_persist_kernel(const __grid_constant__ CUtensorMap tmQ,
           }
         }
         ++k;
+      }
+      if constexpr (kLone) {
+        // ---------------------------------------------- the single tail tile
+        // Prologue: S(0) = Q K_0^T into S buffer 0, S(1) into buffer 1.  Key
+        // step j: P(j) (P also says pair j + 2 landed), before the first P V
+        // "O drained" of tile A's previous item, then P(j) V_j from buffer
+        // j mod 2 and, while tiles remain, S(j + 2) = Q K_{j+2}^T into that
+        // buffer (after the P V that reads it: MMAs run in issue order), one
+        // commit on the buffer's barrier; after the last step also O final.
+        int b = 0, h = 0;
+        bool refresh = false;
+        const int q0 = static_cast<int>(blockIdx.x) < p.n_lone ? lone_q0(b, h, refresh) : p.M;
+        if (ok && q0 < p.M) {
+          auto qk_lone = [&](int buf, uint32_t k_tile) {
+#pragma unroll
+            for (int kk = 0; kk < D / 16; ++kk) {
+              const uint32_t off = (kk >> 2) * kChunkBytes + (kk & 3) * 32;
+              umma_ss(tmem + col_s(buf), sdesc_sw128(sQ + off, 16, 1024), sdesc_sw128(k_tile + off, 16, 1024),
+                      idesc_qk, kk > 0 ? 1u : 0u);
+            }
+          };
+          ok = mbar_wait(lq_full, 0, abort, p.err, p.wait_limit) && mbar_wait(l_full, 0, abort, p.err, p.wait_limit);
+          if (ok) {
+            tc_fence_after();
+            qk_lone(0, sKV + L::kTile);                    // K_0: slot 0's K part
+            umma_commit(l_s);
+          }
+          if (ok && T >= 2) {
+            ok = mbar_wait(l_full + 8, 0, abort, p.err, p.wait_limit);
+            if (ok) {
+              tc_fence_after();
+              qk_lone(1, sKV + 3 * L::kTile);              // K_1: slot 1's K part
+              umma_commit(l_s + 8);
+            }
+          }
+          for (int j = 0; ok && j < T; ++j) {
+            if (p.debug_skip_last_pv && j + 1 == T) { ok = false; break; }   // the softmax's wait for O must expire
+            if (!mbar_wait(l_p + 8 * (j & 1), static_cast<uint32_t>(j >> 1) & 1u, abort, p.err, p.wait_limit) ||
+                (j == 0 && k >= 1 &&
+                 !mbar_wait(bar_o_free, static_cast<uint32_t>(k - 1) & 1u, abort, p.err, p.wait_limit))) {
+              ok = false;
+              break;
+            }
+            tc_fence_after();
+            const int s = j & 1;                           // P(j)'s buffer and pair j + 2's slot
+#pragma unroll
+            for (int kk = 0; kk < 8; ++kk)
+              umma_ts(tmem + col_o(0), tmem + col_s(s) + 64 * (kk >> 2) + (kk & 3) * 8,
+                      sdesc_sw128(sKV + 2 * s * L::kTile + kk * 2048, kChunkBytes, 1024), idesc_pv,
+                      (j > 0 || kk > 0) ? 1u : 0u);
+            if (j + 2 < T) qk_lone(s, sKV + (2 * s + 1) * L::kTile);
+            umma_commit(l_s + 8 * s);
+            if (j + 1 == T) umma_commit(l_o);
+          }
+        }
       }
     }
     __syncwarp();
@@ -1221,6 +1408,95 @@ attn_fwd_persist_kernel(const __grid_constant__ CUtensorMap tmQ,
       ++k;
       if (*stop) break;
     }
+    if constexpr (kLone) {
+      // ------------------------------------------------ the single tail tile
+      // Tile A's warpgroup, after its items: key step j reads S(j) from buffer
+      // j mod 2 (completion j / 2 of that buffer's barrier: the prologue's,
+      // then the commit after key step j - 2), writes P(j) over it and arrives
+      // on P.  A rescale of O must see key step j - 1's P V done: the commit
+      // after it is the next completion of the other buffer (the one that
+      // announces S(j + 1)).  Then O final, and the epilogue in its turn on the
+      // staging buffer.
+      bool has_lone;
+      {
+        int b = 0, h = 0;
+        bool refresh = false;
+        // not after an abort (the walk stops only then; the flag stays set)
+        has_lone = t == 0 && !*abort && static_cast<int>(blockIdx.x) < p.n_lone && lone_q0(b, h, refresh) < p.M;
+      }
+      if (has_lone) {
+        float m_used = -INFINITY;
+        float2 l2 = make_float2(0.f, 0.f);
+        bool failed = false;
+        for (int j = 0; j < T; ++j) {
+          const int s = j & 1;
+          if (!warp_wait(l_s + 8 * s, static_cast<uint32_t>(j >> 1) & 1u, abort, p.err, p.wait_limit)) {
+            failed = true;
+            break;
+          }
+          tc_fence_after();
+          const int valid = j < n_p ? min(kBN, p.P - j * kBN) : min(kBN, p.G - (j - n_p) * kBN);
+          float xs[128];
+          load_scores128(t_lane + col_s(s), valid, xs);
+          const float tm = max128(xs) * sl2;
+          if (j == 0) {
+            m_used = tm;
+          } else if (__any_sync(0xffffffffu, tm > m_used + 8.0f)) {
+            if (!warp_wait(l_s + 8 * (s ^ 1), static_cast<uint32_t>(((j - 1) >> 1) + 1) & 1u, abort, p.err,
+                           p.wait_limit)) {
+              failed = true;
+              break;
+            }
+            tc_fence_after();
+            const float m_new = fmaxf(m_used, tm);
+            const float a = ex2_approx(m_used - m_new);
+            m_used = m_new;
+            l2.x *= a;
+            l2.y *= a;
+            rescale_o(a);
+          }
+          const float2 neg_m = make_float2(-m_used, -m_used);
+          const float2 slv = make_float2(sl2, sl2);
+          float2 acc[2] = {make_float2(0.f, 0.f), make_float2(0.f, 0.f)};
+#pragma unroll
+          for (int q = 0; q < 4; ++q) {
+            uint32_t pk[16];
+#pragma unroll
+            for (int kq = 0; kq < 16; ++kq) {
+              const float2 y = ffma2(make_float2(xs[32 * q + 2 * kq], xs[32 * q + 2 * kq + 1]), slv, neg_m);
+              const float2 pr = make_float2(ex2_approx(y.x), ex2_approx(y.y));
+              acc[kq & 1] = fadd2(acc[kq & 1], pr);
+              pk[kq] = pack_bf16x2(pr.x, pr.y);
+            }
+            tmem_st_16_async(t_lane + col_s(s) + 64 * (q >> 1) + 16 * (q & 1), pk);
+          }
+          tmem_wait_st();
+          l2 = fadd2(l2, fadd2(acc[0], acc[1]));
+          tc_fence_before();
+          mbar_arrive(l_p + 8 * s);
+        }
+        const bool ok = !failed && warp_wait(l_o, 0, abort, p.err, p.wait_limit);
+        tc_fence_after();
+        // (b, h, q0) decoded again from an opaque copy of the CTA index: no
+        // registers held across the key loop
+        int b, h;
+        bool refresh;
+        const int q0 = lone_q0(b, h, refresh, opaque_int(static_cast<int>(blockIdx.x)));
+        const float l_sum = l2.x + l2.y;
+        const int q = q0 + r;
+        const bool live = ok && q < p.M;
+        const int use = 2 * k;                           // tile A's turn on the staging buffer
+        if (use > 0) warp_wait(bar_staged, static_cast<uint32_t>(use - 1) & 1u, abort, p.err, p.wait_limit);
+        stage_o_row<D>(t_lane + colO, stage, r, 1.0f / l_sum);
+        tc_fence_before();
+        mbar_arrive(bar_o_free);                         // O has been read out of TMEM
+        const bool issuer = threadIdx.x == 32 * kWarpSoftmax0;
+        store_o_tile<D>(&tmO, stage, 1u, issuer, ok, h, q0, b, false);
+        if (issuer) mbar_arrive(bar_staged);
+        if (live && p.lse)
+          p.lse[(static_cast<size_t>(b) * p.Hq + h) * p.M + q] = (m_used + log2f(l_sum)) * 0.69314718055994531f;
+      }
+    }
     // the output stores are complete before the CTA exits (they wait on no other thread)
     if (threadIdx.x == 32 * (kWarpSoftmax0 + 4 * t)) bulk_wait_group_all();
     __syncwarp();
@@ -1247,6 +1523,11 @@ attn_fwd_persist_kernel(const __grid_constant__ CUtensorMap tmQ,
     __syncwarp();
     if (q_loads > 0) drain_wait(bar_q_full, static_cast<uint32_t>(q_loads - 1) & 1u, p.wait_limit);
     for (int g = max(0, last_pair - 1); g <= last_pair; ++g) drain_wait(bar_full + 8 * slot_of(g), phase_of(g), p.wait_limit);
+    if constexpr (kLone) {     // the single tail tile's Q load and its latest use of each pair slot
+      if (lone_q) drain_wait(lq_full, 0, p.wait_limit);
+      if (lone_use0 >= 0) drain_wait(l_full, static_cast<uint32_t>(lone_use0) & 1u, p.wait_limit);
+      if (lone_use1 >= 0) drain_wait(l_full + 8, static_cast<uint32_t>(lone_use1) & 1u, p.wait_limit);
+    }
   }
 }
 
@@ -1314,7 +1595,13 @@ int launch_fwd(int kind, cudaLaunchConfig_t lc, const CUtensorMap* m, const Attn
     if (e == cudaSuccess)
       e = cudaFuncSetAttribute(attn_fwd_kernel<D, true, kRw>, cudaFuncAttributeMaxDynamicSharedMemorySize, one);
     if (e == cudaSuccess)
-      e = cudaFuncSetAttribute(attn_fwd_persist_kernel<D, kRw>, cudaFuncAttributeMaxDynamicSharedMemorySize, pers);
+      e = cudaFuncSetAttribute(attn_fwd_persist_kernel<D, kRw, false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                               pers);
+    if constexpr (!kRw) {      // a single-tile tail only in cached steps (no rewrite)
+      if (e == cudaSuccess)
+        e = cudaFuncSetAttribute(attn_fwd_persist_kernel<D, false, true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 pers);
+    }
     if (e != cudaSuccess) return cuda_status(e, "cudaFuncSetAttribute(attention)");
     configured[dev].store(true, std::memory_order_release);
   }
@@ -1323,8 +1610,15 @@ int launch_fwd(int kind, cudaLaunchConfig_t lc, const CUtensorMap* m, const Attn
   cudaError_t e;
   if (kind == kPlanOneTile)
     e = cudaLaunchKernelEx(&lc, attn_fwd_kernel<D, true, kRw>, m[0], m[1], m[2], m[3], m[4], m[5], m[6], m[7], prm);
-  else if (kind == kPlanPersistent)
-    e = cudaLaunchKernelEx(&lc, attn_fwd_persist_kernel<D, kRw>, m[0], m[1], m[2], m[3], m[4], m[5], m[6], m[7], prm);
+  else if (kind == kPlanPersistent && prm.n_lone > 0) {
+    if constexpr (!kRw)
+      e = cudaLaunchKernelEx(&lc, attn_fwd_persist_kernel<D, false, true>, m[0], m[1], m[2], m[3], m[4], m[5], m[6],
+                             m[7], prm);
+    else
+      e = cudaErrorInvalidValue;            // the plan gives refresh launches no single-tile tail
+  } else if (kind == kPlanPersistent)
+    e = cudaLaunchKernelEx(&lc, attn_fwd_persist_kernel<D, kRw, false>, m[0], m[1], m[2], m[3], m[4], m[5], m[6],
+                           m[7], prm);
   else
     e = cudaLaunchKernelEx(&lc, attn_fwd_kernel<D, false, kRw>, m[0], m[1], m[2], m[3], m[4], m[5], m[6], m[7], prm);
   return cuda_status(e, "attention launch");

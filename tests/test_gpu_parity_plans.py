@@ -11,8 +11,9 @@ outputs are of order one and the running-max rescale fires across tiles.
 
 Each case pins the plan the call launches (archer_attn_plan_query on this
 GPU): the two-tile kernel (with and without a last wave of single tiles), the
-persistent kernel for the cached step and the refresh (flags absent and
-mixed), and the flat two-tile refresh with flags over a ragged query range.
+persistent kernel for the cached step (with and without a last wave walked
+as single tiles) and the refresh (flags absent and mixed), and the flat
+two-tile refresh with flags over a ragged query range.
 Per case:
   * at least 8 (sequence, head) pairs, chosen from the launch's work items:
     the first, the last, and items at every depth of the persistent walk
@@ -53,11 +54,11 @@ CASES = {
     # the long-prompt GQA workload's cached step: 896 items, 5.9 per SM
     "persistent_step_gqa_long": ((16, 4096, 512, 28, 4, 128), STEP, None, "persistent", False),
     # the 32-layer trajectory's cached step: 512 items, 3.4 per SM
-    "persistent_step_traj32": ((8, 1024, 512, 32, 32, 128), STEP, None, "persistent", False),
+    "persistent_step_traj32": ((8, 1024, 512, 32, 32, 128), STEP, None, "persistent", True),
     # head_dim 64: 256 items
     "persistent_step_d64": ((8, 1024, 512, 16, 4, 64), STEP, None, "persistent", False),
     # P = 1000: the last prompt key tile holds 104 keys (masked in the softmax), 512 items
-    "persistent_step_ragged_keys": ((8, 1000, 512, 32, 8, 128), STEP, None, "persistent", False),
+    "persistent_step_ragged_keys": ((8, 1000, 512, 32, 8, 128), STEP, None, "persistent", True),
     # P = 0: response-only attention, 896 items of 4 key tiles
     "persistent_step_no_prompt": ((16, 0, 512, 28, 4, 128), STEP, None, "persistent", False),
     # refresh of every sequence: 6 pairs x 32 x 8 = 1536 items
@@ -102,6 +103,8 @@ def sampled_pairs(plan, B, Hq, sms, rng, want=10):
     CTAs; then random items until `want` distinct pairs."""
     units, tiles_x = plan["work_items"], plan["work_items"] // (B * Hq)
     items = [0, units - 1]
+    if plan["single_tail"]:          # the first and a middle item of the last wave (single tiles)
+        items += [units - plan["single_tail"], units - plan["single_tail"] // 2]
     for k in range((units + sms - 1) // sms):
         items.append(min(units - 1, k * sms + (37 * k + 11) % sms))
     pairs = []

@@ -12,7 +12,9 @@ from the planner's rules, with 128-row query tiles and 128-key tiles:
 * two-tile items beyond the SMs: a last wave r = items mod SMs with
   0 < 2 r <= SMs runs as 2 r single-tile CTAs (r extra CTAs);
 * persistent (grid = SMs) when the query ranges are whole tile pairs and
-  either that tail is empty or items >= 3 SMs.
+  either that tail is empty or items >= 3 SMs; in a cached step the tail then
+  runs inside the walk as 2 r single tiles (single_tail = r), in a refresh it
+  is walked in pairs (single_tail = 0).
 """
 import pytest
 
@@ -38,7 +40,7 @@ def test_long_prompt_gqa_cached_step_is_persistent():
 
 def test_long_prompt_gqa_refresh_is_persistent_despite_a_small_last_wave():
     # rows 4608 -> 18 pairs x 28 x 16 = 8064 items; 8064 mod 152 = 8 would be a
-    # tail, but 8064 >= 3 x 152 -> persistent
+    # tail, but 8064 >= 3 x 152 -> persistent, and a refresh walks it in pairs
     for op in (A.ARCHER_PLAN_REFRESH_ALL, A.ARCHER_PLAN_REFRESH_FLAGS):
         p = plan(16, 4096, 512, 28, 4, 128, op=op)
         assert (p["kernel"], p["work_items"], p["grid"], p["single_tail"]) == (A.ARCHER_KERNEL_PERSISTENT, 8064, 152, 0)
@@ -52,10 +54,11 @@ def test_llada_layer_runs_one_tile_ctas_unsplit():
 
 
 def test_32_layer_trajectory_is_persistent_with_3_4_items_per_sm():
-    # 2 pairs x 32 x 8 = 512 items; 512 mod 152 = 56 (a tail) but 512 >= 456
+    # 2 pairs x 32 x 8 = 512 items; 512 mod 152 = 56 (a tail) but 512 >= 456;
+    # the walk takes 456 items in pairs, then 112 single tiles on 112 CTAs
     p = plan(8, 1024, 512, 32, 32, 128)
-    assert (p["kernel"], p["work_items"], p["grid"], p["key_tiles_per_split"]) == (A.ARCHER_KERNEL_PERSISTENT, 512,
-                                                                                   152, 12)
+    assert (p["kernel"], p["work_items"], p["grid"], p["key_tiles_per_split"], p["single_tail"]) == (
+        A.ARCHER_KERNEL_PERSISTENT, 512, 152, 12, 56)
 
 
 def test_key_split_needs_its_workspace():
