@@ -57,10 +57,10 @@ MEASURED_TRAFFIC = {
     # (kernel, workload): DRAM bytes read + written per launch from one ncu capture
     # (dram__bytes_read.sum + dram__bytes_write.sum), valid only while the kernel's
     # sources hash to sha16 (sha256 over the listed files, first 16 hex digits).
-    ("attn_step", "gqa_long"): {"bytes": 209791232 + 37085696, "sha16": "1febb1f8446ec4a2",
+    ("attn_step", "gqa_long"): {"bytes": 209789440 + 36098304, "sha16": "ba834050a6751a49",
                                 "sources": ["attention_kernels.cuh", "attention_step.cu", "archer_device.cuh",
                                             "tmem_ldst.cuh"]},
-    ("attn_refresh", "gqa_long"): {"bytes": 812606208 + 624160512, "sha16": "12870841bac99ddd",
+    ("attn_refresh", "gqa_long"): {"bytes": 813047552 + 623983616, "sha16": "ea665e3400521b8c",
                                    "sources": ["attention_kernels.cuh", "attention_rewrite.cu", "archer_device.cuh",
                                                "tmem_ldst.cuh"]},
     ("scores", "gqa_long"): {"bytes": 2491495424 + 4868096, "sha16": "99cbda7b470f8633",
@@ -842,7 +842,7 @@ def main():
             "speedup_vs_refresh_every_step": value / eager_value,
             "eager_steps_per_s": eager_value,
             "attention": att,
-            "roofline": {"bound": "tensor", "kernel": "attn_fwd_persist_kernel<128, 0> (persistent two-tile, no rewrite)", "launches": "cached step",
+            "roofline": {"bound": "tensor", "kernel": "attn_fwd_persist_kernel<128, 0, 0> (persistent two-tile; no rewrite, no single-tile tail)", "launches": "cached step",
                          "timing": "CUDA events around each cached step's layer loop (host-driven arm), / its launches",
                          "flops_per_launch": flops_step_launch, "achieved": achieved, "peak": peak_tf,
                          "unit": "TFLOP/s", "frac": achieved / peak_tf,
