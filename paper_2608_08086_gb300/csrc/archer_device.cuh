@@ -209,6 +209,16 @@ __device__ __forceinline__ uint64_t sdesc_sw128(uint32_t saddr, uint32_t lbo, ui
   return d;
 }
 
+// The descriptor of the same operand layout `bytes` further on in shared
+// memory (a multiple of 16): only the start-address field (bits 0-13, address
+// >> 4) grows, by bytes >> 4, and it cannot carry out of its 14 bits because
+// shared memory ends below 256 KB.  One 32-bit add instead of rebuilding the
+// descriptor, so that the MMA-issuing thread spends few instructions per MMA.
+__device__ __forceinline__ uint64_t desc_add(uint64_t d, uint32_t bytes) {
+  const uint32_t lo = static_cast<uint32_t>(d) + (bytes >> 4);
+  return (static_cast<uint64_t>(static_cast<uint32_t>(d >> 32)) << 32) | lo;
+}
+
 // Instruction descriptor of tcgen05.mma kind::f16: fp32 accumulator (bits 4-5
 // = 1), bf16 A and B (bits 7-9 = 1, 10-12 = 1), A / B major-ness (bit 15 / 16:
 // 0 = K-major, 1 = MN-major), N >> 3 in bits 17-22, M >> 4 in bits 24-28.

@@ -552,25 +552,29 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
     constexpr uint32_t idesc_qk = idesc_bf16_f32(kBM, kBN, 0, 0);
     constexpr uint32_t idesc_pv = idesc_bf16_f32(kBM, D, 0, 1);
     const int n_tiles = has_b ? 2 : 1;
-    auto issue_qk = [&](int t, uint32_t k_tile) {
-      const uint32_t q_tile = sQ + t * L::kTile;
+    // Operand descriptors built once (Q tile 0; the K and V halves of pair
+    // slot 0); an MMA's own descriptor is one of these plus its offset
+    // (desc_add), so a key step's MMAs cost few instructions.
+    const uint64_t qd0 = sdesc_sw128(sQ, 16, 1024);
+    const uint64_t kd0 = sdesc_sw128(sKV + L::kTile, 16, 1024), vd0 = sdesc_sw128(sKV, kChunkBytes, 1024);
+    auto issue_qk = [&](int t, uint64_t kd) {
+      const uint64_t qd = desc_add(qd0, t * L::kTile);
 #pragma unroll
       for (int kk = 0; kk < D / 16; ++kk) {
         const uint32_t off = (kk >> 2) * kChunkBytes + (kk & 3) * 32;
-        umma_ss(tmem + col_s(t), sdesc_sw128(q_tile + off, 16, 1024), sdesc_sw128(k_tile + off, 16, 1024),
-                idesc_qk, kk > 0 ? 1u : 0u);
+        umma_ss(tmem + col_s(t), desc_add(qd, off), desc_add(kd, off), idesc_qk, kk > 0 ? 1u : 0u);
       }
     };
     // P V over the tile's 128 keys (8 MMAs of K = 16); P of keys
     // [64 h, 64 h + 64) lives in S columns [64 h, 64 h + 32).
-    auto issue_pv = [&](int t, uint32_t v_tile, bool acc) {
+    auto issue_pv = [&](int t, uint64_t vd, bool acc) {
 #pragma unroll
       for (int kk = 0; kk < 8; ++kk)
-        umma_ts(tmem + col_o(t), tmem + col_s(t) + 64 * (kk >> 2) + (kk & 3) * 8,
-                sdesc_sw128(v_tile + kk * 2048, kChunkBytes, 1024), idesc_pv, (acc || kk > 0) ? 1u : 0u);
+        umma_ts(tmem + col_o(t), tmem + col_s(t) + 64 * (kk >> 2) + (kk & 3) * 8, desc_add(vd, kk * 2048), idesc_pv,
+                (acc || kk > 0) ? 1u : 0u);
     };
-    auto v_tile_of = [&](int u) { return sKV + 2 * slot_of(u) * L::kTile; };
-    auto k_tile_of = [&](int u) { return sKV + (2 * slot_of(u) + 1) * L::kTile; };
+    auto v_tile_of = [&](int u) { return desc_add(vd0, slot_of(u) * 2 * L::kTile); };
+    auto k_tile_of = [&](int u) { return desc_add(kd0, slot_of(u) * 2 * L::kTile); };
     auto phase_of = [&](int u) { return static_cast<uint32_t>(use_of(u)) & 1u; };
     if constexpr (kSingle) {
       // One query tile, S double buffered: S(j) in buffer j & 1 (columns
@@ -584,19 +588,18 @@ attn_fwd_kernel(const __grid_constant__ CUtensorMap tmQ,
       // one: O final).  The softmax of tile j + 1 runs meanwhile on the other
       // buffer, so the key step is the longer of one tile's MMAs and one
       // tile's softmax instead of their sum.
-      auto issue_qk1 = [&](int bf, uint32_t k_tile) {
+      auto issue_qk1 = [&](int bf, uint64_t kd) {
 #pragma unroll
         for (int kk = 0; kk < D / 16; ++kk) {
           const uint32_t off = (kk >> 2) * kChunkBytes + (kk & 3) * 32;
-          umma_ss(tmem + col_s(bf), sdesc_sw128(sQ + off, 16, 1024), sdesc_sw128(k_tile + off, 16, 1024),
-                  idesc_qk, kk > 0 ? 1u : 0u);
+          umma_ss(tmem + col_s(bf), desc_add(qd0, off), desc_add(kd, off), idesc_qk, kk > 0 ? 1u : 0u);
         }
       };
-      auto issue_pv1 = [&](int bf, uint32_t v_tile, bool acc) {
+      auto issue_pv1 = [&](int bf, uint64_t vd, bool acc) {
 #pragma unroll
         for (int kk = 0; kk < 8; ++kk)
-          umma_ts(tmem + col_o(0), tmem + col_s(bf) + 64 * (kk >> 2) + (kk & 3) * 8,
-                  sdesc_sw128(v_tile + kk * 2048, kChunkBytes, 1024), idesc_pv, (acc || kk > 0) ? 1u : 0u);
+          umma_ts(tmem + col_o(0), tmem + col_s(bf) + 64 * (kk >> 2) + (kk & 3) * 8, desc_add(vd, kk * 2048),
+                  idesc_pv, (acc || kk > 0) ? 1u : 0u);
       };
       // pairs 0 (K_0) and 1 (V_0, K_1): S(0) and S(1).  Lane 0 alone runs
       // the schedule (single-thread bounded waits); the other lanes wait for
@@ -1196,23 +1199,28 @@ attn_fwd_persist_kernel(const __grid_constant__ CUtensorMap tmQ,
     // also "O final".
     constexpr uint32_t idesc_qk = idesc_bf16_f32(kBM, kBN, 0, 0);
     constexpr uint32_t idesc_pv = idesc_bf16_f32(kBM, D, 0, 1);
-    auto issue_qk = [&](int t, uint32_t k_tile) {
-      const uint32_t q_tile = sQ + t * L::kTile;
+    // Operand descriptors built once: the Q tiles, and the K and V halves of
+    // both pair slots; an MMA's own descriptor is one of these plus its
+    // offset (desc_add), so a key step's 32 MMAs cost few instructions.
+    const uint64_t qd0 = sdesc_sw128(sQ, 16, 1024), qd1 = sdesc_sw128(sQ + L::kTile, 16, 1024);
+    const uint64_t kd0 = sdesc_sw128(sKV + L::kTile, 16, 1024), kd1 = sdesc_sw128(sKV + 3 * L::kTile, 16, 1024);
+    const uint64_t vd0 = sdesc_sw128(sKV, kChunkBytes, 1024), vd1 = sdesc_sw128(sKV + 2 * L::kTile, kChunkBytes, 1024);
+    auto issue_qk = [&](int t, uint64_t kd) {
+      const uint64_t qd = t == 0 ? qd0 : qd1;
 #pragma unroll
       for (int kk = 0; kk < D / 16; ++kk) {
         const uint32_t off = (kk >> 2) * kChunkBytes + (kk & 3) * 32;
-        umma_ss(tmem + col_s(t), sdesc_sw128(q_tile + off, 16, 1024), sdesc_sw128(k_tile + off, 16, 1024),
-                idesc_qk, kk > 0 ? 1u : 0u);
+        umma_ss(tmem + col_s(t), desc_add(qd, off), desc_add(kd, off), idesc_qk, kk > 0 ? 1u : 0u);
       }
     };
-    auto issue_pv = [&](int t, uint32_t v_tile, bool acc) {
+    auto issue_pv = [&](int t, uint64_t vd, bool acc) {
 #pragma unroll
       for (int kk = 0; kk < 8; ++kk)
-        umma_ts(tmem + col_o(t), tmem + col_s(t) + 64 * (kk >> 2) + (kk & 3) * 8,
-                sdesc_sw128(v_tile + kk * 2048, kChunkBytes, 1024), idesc_pv, (acc || kk > 0) ? 1u : 0u);
+        umma_ts(tmem + col_o(t), tmem + col_s(t) + 64 * (kk >> 2) + (kk & 3) * 8, desc_add(vd, kk * 2048), idesc_pv,
+                (acc || kk > 0) ? 1u : 0u);
     };
-    auto v_tile_of = [&](int g) { return sKV + 2 * slot_of(g) * L::kTile; };
-    auto k_tile_of = [&](int g) { return sKV + (2 * slot_of(g) + 1) * L::kTile; };
+    auto v_tile_of = [&](int g) { return slot_of(g) ? vd1 : vd0; };
+    auto k_tile_of = [&](int g) { return slot_of(g) ? kd1 : kd0; };
     bool ok = true;
     if (lane0) {
       int k = 0;
@@ -1262,25 +1270,24 @@ attn_fwd_persist_kernel(const __grid_constant__ CUtensorMap tmQ,
         bool refresh = false;
         const int q0 = static_cast<int>(blockIdx.x) < p.n_lone ? lone_q0(b, h, refresh) : p.M;
         if (ok && q0 < p.M) {
-          auto qk_lone = [&](int buf, uint32_t k_tile) {
+          auto qk_lone = [&](int buf, uint64_t kd) {
 #pragma unroll
             for (int kk = 0; kk < D / 16; ++kk) {
               const uint32_t off = (kk >> 2) * kChunkBytes + (kk & 3) * 32;
-              umma_ss(tmem + col_s(buf), sdesc_sw128(sQ + off, 16, 1024), sdesc_sw128(k_tile + off, 16, 1024),
-                      idesc_qk, kk > 0 ? 1u : 0u);
+              umma_ss(tmem + col_s(buf), desc_add(qd0, off), desc_add(kd, off), idesc_qk, kk > 0 ? 1u : 0u);
             }
           };
           ok = mbar_wait(lq_full, 0, abort, p.err, p.wait_limit) && mbar_wait(l_full, 0, abort, p.err, p.wait_limit);
           if (ok) {
             tc_fence_after();
-            qk_lone(0, sKV + L::kTile);                    // K_0: slot 0's K part
+            qk_lone(0, kd0);                               // K_0: slot 0's K part
             umma_commit(l_s);
           }
           if (ok && T >= 2) {
             ok = mbar_wait(l_full + 8, 0, abort, p.err, p.wait_limit);
             if (ok) {
               tc_fence_after();
-              qk_lone(1, sKV + 3 * L::kTile);              // K_1: slot 1's K part
+              qk_lone(1, kd1);                             // K_1: slot 1's K part
               umma_commit(l_s + 8);
             }
           }
@@ -1297,9 +1304,9 @@ attn_fwd_persist_kernel(const __grid_constant__ CUtensorMap tmQ,
 #pragma unroll
             for (int kk = 0; kk < 8; ++kk)
               umma_ts(tmem + col_o(0), tmem + col_s(s) + 64 * (kk >> 2) + (kk & 3) * 8,
-                      sdesc_sw128(sKV + 2 * s * L::kTile + kk * 2048, kChunkBytes, 1024), idesc_pv,
+                      desc_add(s ? vd1 : vd0, kk * 2048), idesc_pv,
                       (j > 0 || kk > 0) ? 1u : 0u);
-            if (j + 2 < T) qk_lone(s, sKV + (2 * s + 1) * L::kTile);
+            if (j + 2 < T) qk_lone(s, s ? kd1 : kd0);
             umma_commit(l_s + 8 * s);
             if (j + 1 == T) umma_commit(l_o);
           }
