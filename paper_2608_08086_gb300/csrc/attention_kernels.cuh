@@ -1021,10 +1021,11 @@ attn_fwd_persist_kernel(const __grid_constant__ CUtensorMap tmQ,
     //           P V read pair g0 - 1, whose slot pair g0 + 1 takes); then the
     //           gate, without which this item's prologue cannot complete S_B.
     //   u >= 2  S_B completion g - 2 (the prologue or key step u - 3, the last
-    //           reads of pair g - 2); then pair g - 1's arrival on P_A, without
-    //           which key step u - 2 cannot complete S_B.
+    //           reads of pair g - 2); then pair g - 1's arrival on P_A (its
+    //           landing seen before that poll), without which key step u - 2
+    //           cannot complete S_B.
     //   end     S_B completion g0 + T - 1 (key step T - 2, or the prologue), then
-    //           the arrival for the item's last pair.
+    //           the arrival for the item's last pair (landed, seen before).
     // An arrival on P_A must fall in the phase it is meant for: each follows an
     // S_B completion that the MMA warp committed after waiting for the phase
     // before.
@@ -1039,9 +1040,12 @@ attn_fwd_persist_kernel(const __grid_constant__ CUtensorMap tmQ,
       const CUtensorMap* mKp = refresh ? &tmKpR : &tmKpC;
       const CUtensorMap* mVp = refresh ? &tmVpR : &tmVpC;
       const int g0 = k * (T + 1);
-      // pair v landed -> its arrival on P_A
-      auto arrive_landed = [&](int v) {
-        if (!warp_wait(bar_full + 8 * slot_of(v), phase_of(v), abort, p.err, p.wait_limit)) return false;
+      // Pair v's landing is waited for before the S_B poll that its arrival
+      // on P_A must follow, so that the arrival comes right after that poll
+      // (key step j's softmax warps arrive on P_A soon after S_B's completion
+      // for key step j - 1).
+      auto landed = [&](int v) { return warp_wait(bar_full + 8 * slot_of(v), phase_of(v), abort, p.err, p.wait_limit); };
+      auto arrive = [&]() {
         if (lane0) mbar_arrive(bar_p_full);
         __syncwarp();
         return true;
@@ -1057,8 +1061,8 @@ attn_fwd_persist_kernel(const __grid_constant__ CUtensorMap tmQ,
           __syncwarp();
           gate_pending = false;
         } else if (u >= 2) {
-          if (!warp_wait(bar_s_full + 8, static_cast<uint32_t>(g - 2) & 1u, abort, p.err, p.wait_limit) ||
-              !arrive_landed(g - 1)) {
+          if (!landed(g - 1) ||
+              !warp_wait(bar_s_full + 8, static_cast<uint32_t>(g - 2) & 1u, abort, p.err, p.wait_limit) || !arrive()) {
             ok = false;
             break;
           }
@@ -1102,8 +1106,8 @@ attn_fwd_persist_kernel(const __grid_constant__ CUtensorMap tmQ,
       }
       if (!ok) break;
       // the item's end: S_B completion g0 + T - 1, then the last pair's arrival
-      if (!warp_wait(bar_s_full + 8, static_cast<uint32_t>(g0 + T - 1) & 1u, abort, p.err, p.wait_limit) ||
-          !arrive_landed(g0 + T)) {
+      if (!landed(g0 + T) ||
+          !warp_wait(bar_s_full + 8, static_cast<uint32_t>(g0 + T - 1) & 1u, abort, p.err, p.wait_limit) || !arrive()) {
         ok = false;
         break;
       }
