@@ -57,10 +57,10 @@ MEASURED_TRAFFIC = {
     # (kernel, workload): DRAM bytes read + written per launch from one ncu capture
     # (dram__bytes_read.sum + dram__bytes_write.sum), valid only while the kernel's
     # sources hash to sha16 (sha256 over the listed files, first 16 hex digits).
-    ("attn_step", "gqa_long"): {"bytes": 209789440 + 36098304, "sha16": "ba834050a6751a49",
+    ("attn_step", "gqa_long"): {"bytes": 209790720 + 37077504, "sha16": "7342f15723f3de85",
                                 "sources": ["attention_kernels.cuh", "attention_step.cu", "archer_device.cuh",
                                             "tmem_ldst.cuh"]},
-    ("attn_refresh", "gqa_long"): {"bytes": 813047552 + 623983616, "sha16": "ea665e3400521b8c",
+    ("attn_refresh", "gqa_long"): {"bytes": 813386752 + 624214016, "sha16": "9e76c03377f258e1",
                                    "sources": ["attention_kernels.cuh", "attention_rewrite.cu", "archer_device.cuh",
                                                "tmem_ldst.cuh"]},
     ("scores", "gqa_long"): {"bytes": 2491495424 + 4868096, "sha16": "99cbda7b470f8633",
