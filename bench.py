@@ -63,7 +63,7 @@ MEASURED_TRAFFIC = {
     ("attn_refresh", "gqa_long"): {"bytes": 813386752 + 624214016, "sha16": "9e76c03377f258e1",
                                    "sources": ["attention_kernels.cuh", "attention_rewrite.cu", "archer_device.cuh",
                                                "tmem_ldst.cuh"]},
-    ("scores", "gqa_long"): {"bytes": 2491495424 + 4868096, "sha16": "99cbda7b470f8633",
+    ("scores", "gqa_long"): {"bytes": 2491648000 + 4957440, "sha16": "a5463d9160dc1f66",
                              "sources": ["decode_scores.cu", "archer_device.cuh"]},
 }
 
