@@ -191,6 +191,19 @@ __device__ __forceinline__ bool warp_wait(uint32_t bar, uint32_t parity, volatil
 
 // v, as a value the compiler cannot see through: what is computed from it is
 // recomputed there, not kept alive from an earlier computation of the same.
+// A descriptor the compiler cannot see through: the MMA-issuing thread starts
+// each batch from an opaque copy of its base descriptor, placed after the
+// wait that precedes the batch, and steps to the next MMA's operand with one
+// add after each MMA.  Otherwise the compiler computes a key step's
+// descriptors ahead of that wait, on the issuing warp's critical path (the
+// warp shares its SM sub-partition with two softmax warps, so every
+// instruction there costs several cycles), instead of between MMAs, where
+// they overlap the tensor core's work.
+__device__ __forceinline__ uint64_t opaque_desc(uint64_t v) {
+  uint64_t r;
+  asm volatile("mov.b64 %0, %1;" : "=l"(r) : "l"(v));
+  return r;
+}
 __device__ __forceinline__ int opaque_int(int v) {
   asm volatile("" : "+r"(v));
   return v;
@@ -1209,19 +1222,25 @@ attn_fwd_persist_kernel(const __grid_constant__ CUtensorMap tmQ,
     const uint64_t qd0 = sdesc_sw128(sQ, 16, 1024), qd1 = sdesc_sw128(sQ + L::kTile, 16, 1024);
     const uint64_t kd0 = sdesc_sw128(sKV + L::kTile, 16, 1024), kd1 = sdesc_sw128(sKV + 3 * L::kTile, 16, 1024);
     const uint64_t vd0 = sdesc_sw128(sKV, kChunkBytes, 1024), vd1 = sdesc_sw128(sKV + 2 * L::kTile, kChunkBytes, 1024);
+    // Each batch's descriptors step from an opaque copy of its base, one add
+    // after each MMA (see opaque_desc).
     auto issue_qk = [&](int t, uint64_t kd) {
-      const uint64_t qd = t == 0 ? qd0 : qd1;
+      uint64_t qa = opaque_desc(t == 0 ? qd0 : qd1), ka = opaque_desc(kd);
 #pragma unroll
       for (int kk = 0; kk < D / 16; ++kk) {
-        const uint32_t off = (kk >> 2) * kChunkBytes + (kk & 3) * 32;
-        umma_ss(tmem + col_s(t), desc_add(qd, off), desc_add(kd, off), idesc_qk, kk > 0 ? 1u : 0u);
+        umma_ss(tmem + col_s(t), qa, ka, idesc_qk, kk > 0 ? 1u : 0u);
+        const uint32_t step = (kk & 3) == 3 ? kChunkBytes - 96 : 32;   // to (kk + 1): 32 B, or the next chunk
+        qa = desc_add(qa, step);
+        ka = desc_add(ka, step);
       }
     };
     auto issue_pv = [&](int t, uint64_t vd, bool acc) {
+      uint64_t va = opaque_desc(vd);
 #pragma unroll
-      for (int kk = 0; kk < 8; ++kk)
-        umma_ts(tmem + col_o(t), tmem + col_s(t) + 64 * (kk >> 2) + (kk & 3) * 8, desc_add(vd, kk * 2048), idesc_pv,
-                (acc || kk > 0) ? 1u : 0u);
+      for (int kk = 0; kk < 8; ++kk) {
+        umma_ts(tmem + col_o(t), tmem + col_s(t) + 64 * (kk >> 2) + (kk & 3) * 8, va, idesc_pv, (acc || kk > 0) ? 1u : 0u);
+        va = desc_add(va, 2048);
+      }
     };
     auto v_tile_of = [&](int g) { return slot_of(g) ? vd1 : vd0; };
     auto k_tile_of = [&](int g) { return slot_of(g) ? kd1 : kd0; };
@@ -1275,10 +1294,13 @@ attn_fwd_persist_kernel(const __grid_constant__ CUtensorMap tmQ,
         const int q0 = static_cast<int>(blockIdx.x) < p.n_lone ? lone_q0(b, h, refresh) : p.M;
         if (ok && q0 < p.M) {
           auto qk_lone = [&](int buf, uint64_t kd) {
+            uint64_t qa = opaque_desc(qd0), ka = opaque_desc(kd);
 #pragma unroll
             for (int kk = 0; kk < D / 16; ++kk) {
-              const uint32_t off = (kk >> 2) * kChunkBytes + (kk & 3) * 32;
-              umma_ss(tmem + col_s(buf), desc_add(qd0, off), desc_add(kd, off), idesc_qk, kk > 0 ? 1u : 0u);
+              umma_ss(tmem + col_s(buf), qa, ka, idesc_qk, kk > 0 ? 1u : 0u);
+              const uint32_t step = (kk & 3) == 3 ? kChunkBytes - 96 : 32;
+              qa = desc_add(qa, step);
+              ka = desc_add(ka, step);
             }
           };
           ok = mbar_wait(lq_full, 0, abort, p.err, p.wait_limit) && mbar_wait(l_full, 0, abort, p.err, p.wait_limit);
@@ -1305,11 +1327,13 @@ attn_fwd_persist_kernel(const __grid_constant__ CUtensorMap tmQ,
             }
             tc_fence_after();
             const int s = j & 1;                           // P(j)'s buffer and pair j + 2's slot
+            uint64_t va = opaque_desc(s ? vd1 : vd0);
 #pragma unroll
-            for (int kk = 0; kk < 8; ++kk)
-              umma_ts(tmem + col_o(0), tmem + col_s(s) + 64 * (kk >> 2) + (kk & 3) * 8,
-                      desc_add(s ? vd1 : vd0, kk * 2048), idesc_pv,
+            for (int kk = 0; kk < 8; ++kk) {
+              umma_ts(tmem + col_o(0), tmem + col_s(s) + 64 * (kk >> 2) + (kk & 3) * 8, va, idesc_pv,
                       (j > 0 || kk > 0) ? 1u : 0u);
+              va = desc_add(va, 2048);
+            }
             if (j + 2 < T) qk_lone(s, s ? kd1 : kd0);
             umma_commit(l_s + 8 * s);
             if (j + 1 == T) umma_commit(l_o);
