@@ -57,10 +57,10 @@ MEASURED_TRAFFIC = {
     # (kernel, workload): DRAM bytes read + written per launch from one ncu capture
     # (dram__bytes_read.sum + dram__bytes_write.sum), valid only while the kernel's
     # sources hash to sha16 (sha256 over the listed files, first 16 hex digits).
-    ("attn_step", "gqa_long"): {"bytes": 209795072 + 36811520, "sha16": "0e32f050c84952ab",
+    ("attn_step", "gqa_long"): {"bytes": 209805312 + 37449472, "sha16": "690d916fd55f72d2",
                                 "sources": ["attention_kernels.cuh", "attention_step.cu", "archer_device.cuh",
                                             "tmem_ldst.cuh"]},
-    ("attn_refresh", "gqa_long"): {"bytes": 812352768 + 624469248, "sha16": "1c5ed543c224f612",
+    ("attn_refresh", "gqa_long"): {"bytes": 811404288 + 624242432, "sha16": "7c2d92b506cdc695",
                                    "sources": ["attention_kernels.cuh", "attention_rewrite.cu", "archer_device.cuh",
                                                "tmem_ldst.cuh"]},
     ("scores", "gqa_long"): {"bytes": 2491648000 + 4957440, "sha16": "a5463d9160dc1f66",
