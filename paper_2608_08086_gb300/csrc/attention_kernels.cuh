@@ -1060,6 +1060,11 @@ attn_fwd_persist_kernel(const __grid_constant__ CUtensorMap tmQ,
       const CUtensorMap* mKp = refresh ? &tmKpR : &tmKpC;
       const CUtensorMap* mVp = refresh ? &tmVpR : &tmVpC;
       const int g0 = k * (T + 1);
+      // deep L2 prefetch of the K/V stream (below): cached steps of
+      // one-query-head-per-kv-head shapes, by the first item of the head, in
+      // the single-tile-tail instantiation only (carrying the code, even
+      // untaken, slowed the kernel that walks the long-prompt GQA step)
+      const bool lead = kLone && p.Hq == p.Hkv && (x % p.tiles_x) == 0;
       // Pair v's landing is waited for before the S_B poll that its arrival
       // on P_A must follow, so that the arrival comes right after that poll
       // (key step j's softmax warps arrive on P_A soon after S_B's completion
@@ -1111,6 +1116,22 @@ attn_fwd_persist_kernel(const __grid_constant__ CUtensorMap tmQ,
             const uint32_t dst = sKV + (2 * slot + part) * L::kTile;
             for (int c = 0; c < L::kChunks; ++c)
               tma_load_4d(dst + c * kChunkBytes, map, bar_full + 8 * slot, c * 64, kvh, row, b);
+          }
+          // the K/V tiles of pair g + 2 (V_{u+1}, K_{u+2}) into L2 now, two
+          // key steps before their own load, where each kv head feeds a
+          // single query head: its K/V stream then comes from DRAM for one
+          // pair of items (with several query heads per kv head the tiles are
+          // read by many items at once and mostly hit L2, and the prefetch
+          // instructions only delay the producer's arrivals)
+          if constexpr (kLone) {
+            for (int part = 0; lead && part < 2; ++part) {
+              const int j = part == 0 ? u + 1 : u + 2;
+              if (j >= T) continue;
+              const bool in_prompt = j < n_p;
+              const int row = in_prompt ? j * kBN : (j - n_p) * kBN;
+              const CUtensorMap* map = in_prompt ? (part == 0 ? mVp : mKp) : (part == 0 ? &tmVg : &tmKg);
+              for (int c = 0; c < L::kChunks; ++c) tma_prefetch_4d(map, c * 64, kvh, row, b);
+            }
           }
           if (u == max(0, T - 2 - (static_cast<int>(blockIdx.x) & 3))) {
             if constexpr (kLone) {
