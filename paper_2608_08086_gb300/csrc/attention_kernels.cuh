@@ -942,9 +942,10 @@ attn_fwd_persist_kernel(const __grid_constant__ CUtensorMap tmQ,
   };
 
   // A launch without refresh flags (a cached step) waits for the grid it
-  // depends on only after its set-up; its inputs are not that grid's
-  // outputs, and an L2 prefetch is only a hint that L2 keeps coherent with
-  // any write.  So the producer lane prefetches the CTA's first item into L2
+  // depends on only after its set-up.  Its loads all come after that wait;
+  // an L2 prefetch is only a hint, and L2 stays coherent with whatever the
+  // previous grid still writes (the first layer's inputs can be its
+  // outputs).  So the producer lane prefetches the CTA's first item into L2
   // right away, while the previous launch ends: every launch of a step reads
   // a layer's K/V afresh from DRAM.
   if (!p.flags && threadIdx.x == 32 * kWarpProducer) prefetch_item(blockIdx.x);
