@@ -57,10 +57,10 @@ MEASURED_TRAFFIC = {
     # (kernel, workload): DRAM bytes read + written per launch from one ncu capture
     # (dram__bytes_read.sum + dram__bytes_write.sum), valid only while the kernel's
     # sources hash to sha16 (sha256 over the listed files, first 16 hex digits).
-    ("attn_step", "gqa_long"): {"bytes": 209796096 + 36525056, "sha16": "56d67f9dcdec60e5",
+    ("attn_step", "gqa_long"): {"bytes": 209797120 + 37160448, "sha16": "bba83f495a267f1c",
                                 "sources": ["attention_kernels.cuh", "attention_step.cu", "archer_device.cuh",
                                             "tmem_ldst.cuh"]},
-    ("attn_refresh", "gqa_long"): {"bytes": 811278080 + 624307200, "sha16": "99289fb373c3192b",
+    ("attn_refresh", "gqa_long"): {"bytes": 812074496 + 624359680, "sha16": "8dfd63cb241930e0",
                                    "sources": ["attention_kernels.cuh", "attention_rewrite.cu", "archer_device.cuh",
                                                "tmem_ldst.cuh"]},
     ("scores", "gqa_long"): {"bytes": 2491648000 + 4957440, "sha16": "a5463d9160dc1f66",
