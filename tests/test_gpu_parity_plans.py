@@ -57,6 +57,9 @@ CASES = {
     "persistent_step_traj32": ((8, 1024, 512, 32, 32, 128), STEP, None, "persistent", True),
     # head_dim 64: 256 items
     "persistent_step_d64": ((8, 1024, 512, 16, 4, 64), STEP, None, "persistent", False),
+    # head_dim 64, one query head per kv head, 512 items: the single-tile tail
+    # and the K/V stream's L2 prefetch in the head_dim 64 instantiation
+    "persistent_step_d64_mha_tail": ((4, 1024, 512, 64, 64, 64), STEP, None, "persistent", True),
     # P = 1000: the last prompt key tile holds 104 keys (masked in the softmax), 512 items
     "persistent_step_ragged_keys": ((8, 1000, 512, 32, 8, 128), STEP, None, "persistent", True),
     # P = 0: response-only attention, 896 items of 4 key tiles
